@@ -1,0 +1,265 @@
+/* Reference oracle for stale-synchronous MF-SGD: plain fp64 C, single thread.
+ *
+ * TEST INFRASTRUCTURE ONLY (tests, smoke check, CPU baseline of the bench).
+ * See esspt_oracle.h for the per-clock semantics and the paper passages they
+ * follow.  Readings of passages the paper leaves open:
+ *   - clocks are 1-based; version v is the table after clocks 1..v; a read at
+ *     clock c must see every update of clocks 1..c-1-s, so
+ *     max(0, c-1-s) <= v_p(c) <= c-1, and s = 0 gives v = c-1: the BSP
+ *     clock differential v - c = -1 of Fig. 1;
+ *   - SSP lazy pull refreshes a worker's whole cached table only when it
+ *     would otherwise break the bound ("waits until the last minute",
+ *     Sec. 2.2), at a seeded per-worker phase phi_p in [0, s];
+ *   - ESSP eager push: the server's push of version c-1 reaches worker p
+ *     after a delay of delta_{p,c} ~ Geometric(p) clocks clamped to
+ *     [0, min(max_delay, s)]; the read version never goes backwards;
+ *   - all entries of a worker in one clock read the same version and both
+ *     updates use the old L_i and R_j (no read-my-writes, Sec. 3 footnote).
+ */
+#include "esspt_oracle.h"
+
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORC_STREAM_PHASE 101u
+#define ORC_STREAM_DELAY 102u
+
+/* SplitMix64 (Steele, Lea and Flood, OOPSLA 2014): output n of a sequence
+ * with initial state s0 is mix(s0 + n * 0x9E3779B97F4A7C15). */
+static uint64_t orc_mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+uint64_t orc_ctr_u64(uint64_t seed, uint64_t stream, uint64_t index) {
+  uint64_t s0 = orc_mix64(seed) ^ orc_mix64(stream);
+  return orc_mix64(s0 + (index + 1u) * 0x9E3779B97F4A7C15ull);
+}
+
+/* Map a draw to [0, n) by the multiply-high of its top 32 bits. */
+static uint32_t orc_below(uint64_t h, uint32_t n) {
+  return (uint32_t)(((h >> 32) * (uint64_t)n) >> 32);
+}
+
+struct orc_state {
+  orc_config cfg;
+  int64_t n_obs;
+  const int32_t* i;
+  const int32_t* j;
+  const float* D;
+  const uint8_t* mb;
+  const int32_t* w;
+  int64_t rows;     /* N + M */
+  int32_t nslots;   /* versions held */
+  double* tables;   /* nslots * rows * K */
+  int32_t version;  /* newest complete version */
+  int32_t* v_prev;  /* read versions of the last clock (P) */
+  double* delta;    /* rows * K */
+  int64_t* count;   /* rows, entries per row in this clock */
+};
+
+static double* orc_slot(const orc_state* st, int32_t version) {
+  int64_t slot = st->cfg.keep_all ? version : version % st->nslots;
+  return st->tables + slot * st->rows * st->cfg.K;
+}
+
+static int orc_holds(const orc_state* st, int32_t version) {
+  if (version < 0 || version > st->version) return 0;
+  if (st->cfg.keep_all) return 1;
+  return version > st->version - st->nslots;
+}
+
+int orc_schedule_rule(const orc_config* cfg, int32_t c, const int32_t* v_prev, int32_t* v_out) {
+  int32_t lo = c - 1 - cfg->s;
+  if (lo < 0) lo = 0;
+  for (int32_t p = 0; p < cfg->P; ++p) {
+    int32_t v;
+    if (cfg->model == ORC_SSP_LAZY) {
+      /* Lazy pull: staleness (c-1) - v cycles 0, 1, ..., s with phase phi_p. */
+      int32_t phi = 0;
+      if (cfg->phased) phi = (int32_t)orc_below(orc_ctr_u64(cfg->seed, ORC_STREAM_PHASE, (uint64_t)p), (uint32_t)(cfg->s + 1));
+      v = (c - 1) - ((c - 1 + phi) % (cfg->s + 1));
+      if (v < 0) v = 0;
+    } else if (cfg->model == ORC_ESSP_EAGER) {
+      /* Eager push: delay = number of failures before the first success of a
+       * Bernoulli(essp_p) sequence, by inverse CDF on a 32-bit uniform u:
+       * delay >= k  iff  u < floor((1-essp_p)^k * 2^32). */
+      int32_t dmax = cfg->essp_max_delay < cfg->s ? cfg->essp_max_delay : cfg->s;
+      uint32_t u = (uint32_t)(orc_ctr_u64(cfg->seed, ORC_STREAM_DELAY, ((uint64_t)(uint32_t)c << 32) | (uint32_t)p) >> 32);
+      double q = 1.0, fail = 1.0 - cfg->essp_p;
+      int32_t delay = 0;
+      for (int32_t k = 1; k <= dmax; ++k) {
+        q *= fail;
+        uint32_t thr = (uint32_t)floor(q * 4294967296.0);
+        if (u < thr) delay = k;
+      }
+      v = c - 1 - delay;
+      if (v_prev != NULL && v_prev[p] > v) v = v_prev[p];
+      if (v < 0) v = 0;
+    } else {
+      return -1;
+    }
+    v_out[p] = v;
+  }
+  for (int32_t p = 0; p < cfg->P; ++p)
+    if (v_out[p] < lo || v_out[p] > c - 1) return -1;
+  return 0;
+}
+
+orc_state* orc_create(const orc_config* cfg, int64_t n_obs, const int32_t* i, const int32_t* j,
+                      const float* D, const uint8_t* minibatch, const int32_t* user_worker,
+                      const float* L0, const float* R0) {
+  if (!cfg || cfg->n_users <= 0 || cfg->n_items <= 0 || cfg->K <= 0 || cfg->P <= 0 || cfg->s < 0 ||
+      cfg->F <= 0 || n_obs < 0 || cfg->model < 0 || cfg->model > ORC_EXTERNAL)
+    return NULL;
+  orc_state* st = (orc_state*)calloc(1, sizeof(orc_state));
+  if (!st) return NULL;
+  st->cfg = *cfg;
+  st->n_obs = n_obs;
+  st->i = i;
+  st->j = j;
+  st->D = D;
+  st->mb = minibatch;
+  st->w = user_worker;
+  st->rows = cfg->n_users + cfg->n_items;
+  /* s+1 readable versions plus the one being written. */
+  st->nslots = cfg->keep_all ? 1 : cfg->s + 2;
+  int64_t K = cfg->K;
+  st->tables = (double*)calloc((size_t)(st->nslots * st->rows * K), sizeof(double));
+  st->v_prev = (int32_t*)calloc((size_t)cfg->P, sizeof(int32_t));
+  st->delta = (double*)calloc((size_t)(st->rows * K), sizeof(double));
+  st->count = (int64_t*)calloc((size_t)st->rows, sizeof(int64_t));
+  if (!st->tables || !st->v_prev || !st->delta || !st->count) {
+    orc_destroy(st);
+    return NULL;
+  }
+  double* x0 = st->tables;
+  for (int64_t r = 0; r < cfg->n_users; ++r)
+    for (int64_t q = 0; q < K; ++q) x0[r * K + q] = (double)L0[r * K + q];
+  for (int64_t r = 0; r < cfg->n_items; ++r)
+    for (int64_t q = 0; q < K; ++q) x0[(cfg->n_users + r) * K + q] = (double)R0[r * K + q];
+  st->version = 0;
+  return st;
+}
+
+void orc_destroy(orc_state* st) {
+  if (!st) return;
+  free(st->tables);
+  free(st->v_prev);
+  free(st->delta);
+  free(st->count);
+  free(st);
+}
+
+static int orc_grow(orc_state* st) {
+  /* keep_all: one more version slot. */
+  size_t per = (size_t)(st->rows * st->cfg.K);
+  double* t = (double*)realloc(st->tables, (size_t)(st->nslots + 1) * per * sizeof(double));
+  if (!t) return -1;
+  st->tables = t;
+  st->nslots += 1;
+  return 0;
+}
+
+int orc_clock(orc_state* st, const int32_t* v_ext) {
+  const orc_config* cfg = &st->cfg;
+  const int64_t K = cfg->K, N = cfg->n_users;
+  int32_t c = st->version + 1;
+  int32_t* v = (int32_t*)malloc((size_t)cfg->P * sizeof(int32_t));
+  if (!v) return -2;
+
+  /* 1. Read versions. */
+  if (cfg->model == ORC_EXTERNAL) {
+    int32_t lo = c - 1 - cfg->s < 0 ? 0 : c - 1 - cfg->s;
+    for (int32_t p = 0; p < cfg->P; ++p) {
+      v[p] = v_ext[p];
+      if (v[p] < lo || v[p] > c - 1) {
+        free(v);
+        return -1;
+      }
+    }
+  } else if (orc_schedule_rule(cfg, c, st->v_prev, v) != 0) {
+    free(v);
+    return -1;
+  }
+  if (cfg->keep_all && orc_grow(st) != 0) {
+    free(v);
+    return -2;
+  }
+
+  /* 2. Deltas of every entry of minibatch b, each at its worker's version. */
+  memset(st->delta, 0, (size_t)(st->rows * K) * sizeof(double));
+  memset(st->count, 0, (size_t)st->rows * sizeof(int64_t));
+  const uint8_t b = (uint8_t)((c - 1) % cfg->F);
+  for (int64_t k = 0; k < st->n_obs; ++k) {
+    if (st->mb[k] != b) continue;
+    int64_t ui = st->i[k], ij = st->j[k];
+    int32_t p = st->w[ui];
+    const double* x = orc_slot(st, v[p]);
+    const double* Li = x + ui * K;
+    const double* Rj = x + (N + ij) * K;
+    double dot = 0.0;
+    for (int64_t q = 0; q < K; ++q) dot += Li[q] * Rj[q];
+    double e = (double)st->D[k] - dot;
+    double* dL = st->delta + ui * K;
+    double* dR = st->delta + (N + ij) * K;
+    for (int64_t q = 0; q < K; ++q) {
+      dL[q] += cfg->eta * (e * Rj[q] - cfg->lambda * Li[q]);
+      dR[q] += cfg->eta * (e * Li[q] - cfg->lambda * Rj[q]);
+    }
+    st->count[ui] += 1;
+    st->count[N + ij] += 1;
+  }
+
+  /* 3. Clock() merge into version c. */
+  const double* prev = orc_slot(st, c - 1);
+  st->version = c; /* slot of c is now addressable */
+  double* next = orc_slot(st, c);
+  for (int64_t r = 0; r < st->rows; ++r) {
+    double scale = 1.0;
+    if (cfg->cap > 0 && st->count[r] > cfg->cap) scale = (double)cfg->cap / (double)st->count[r];
+    for (int64_t q = 0; q < K; ++q) next[r * K + q] = prev[r * K + q] + scale * st->delta[r * K + q];
+  }
+  memcpy(st->v_prev, v, (size_t)cfg->P * sizeof(int32_t));
+  free(v);
+  return 0;
+}
+
+int32_t orc_version(const orc_state* st) { return st->version; }
+
+int orc_schedule(const orc_state* st, int32_t* v_out) {
+  if (st->version < 1) return -1;
+  memcpy(v_out, st->v_prev, (size_t)st->cfg.P * sizeof(int32_t));
+  return 0;
+}
+
+int orc_table(const orc_state* st, int32_t version, double* out) {
+  if (!orc_holds(st, version)) return -1;
+  memcpy(out, orc_slot(st, version), (size_t)(st->rows * st->cfg.K) * sizeof(double));
+  return 0;
+}
+
+int orc_objective(const orc_state* st, int32_t version, double* sq, double* pen) {
+  if (!orc_holds(st, version)) return -1;
+  const int64_t K = st->cfg.K, N = st->cfg.n_users;
+  const double* x = orc_slot(st, version);
+  double s1 = 0.0, s2 = 0.0;
+  for (int64_t k = 0; k < st->n_obs; ++k) {
+    const double* Li = x + (int64_t)st->i[k] * K;
+    const double* Rj = x + (N + st->j[k]) * K;
+    double dot = 0.0, nl = 0.0, nr = 0.0;
+    for (int64_t q = 0; q < K; ++q) {
+      dot += Li[q] * Rj[q];
+      nl += Li[q] * Li[q];
+      nr += Rj[q] * Rj[q];
+    }
+    double e = (double)st->D[k] - dot;
+    s1 += e * e;
+    s2 += e * e + st->cfg.lambda * (nl + nr);
+  }
+  *sq = s1;
+  *pen = s2;
+  return 0;
+}

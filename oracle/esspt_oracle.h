@@ -1,0 +1,92 @@
+/* Reference oracle for one clock of stale-synchronous MF-SGD.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This is a plain, slow, single-threaded fp64 CPU
+ * restatement of the paper's per-clock semantics.  It exists to check the
+ * CUDA library; only the test suite, the smoke check and the benchmark's CPU
+ * baseline may load it.  It shares no code, header or constant with the CUDA
+ * library.
+ *
+ * What one clock c (1-based) computes, producing table version c:
+ *   1. the read version v_p(c) of every worker p (Sec. 2.2 SSP condition;
+ *      Sec. 3 formal SSP bound; Sec. 4 READ guarantee and server push),
+ *      checked against max(0, c-1-s) <= v_p(c) <= c-1;
+ *   2. for every observed entry (i, j) of minibatch b = (c-1) mod F, owned by
+ *      worker p = w(i): e = D_ij - L_i . R_j at version v_p(c), and the
+ *      Sec. 3.1 updates  dL_i += eta (e R_j - lambda L_i),
+ *                         dR_j += eta (e L_i - lambda R_j),
+ *      both from the same read version (no read-my-writes, Sec. 3 footnote);
+ *   3. the Clock() merge X[c] = X[c-1] + scale (.) sum of deltas (additive
+ *      updates, Sec. 2.1; coalesced per clock, Sec. 4), where scale is 1
+ *      unless the hot-row step cap C is on: then row r's summed delta is
+ *      scaled by min(1, C / n_r), n_r = entries of row r in this clock.
+ *
+ * Tables are (n_users + n_items) rows of K doubles: user rows 0..N-1 are L,
+ * item rows N..N+M-1 are R (one row per item, the transpose of the paper's
+ * column R_{*j}).
+ */
+#ifndef ESSPT_ORACLE_H
+#define ESSPT_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum { ORC_SSP_LAZY = 0, ORC_ESSP_EAGER = 1, ORC_EXTERNAL = 2 };
+
+typedef struct {
+  int64_t n_users;     /* N */
+  int64_t n_items;     /* M */
+  int32_t K;           /* rank */
+  int32_t P;           /* workers */
+  int32_t s;           /* staleness bound */
+  int32_t F;           /* minibatches per pass; clock c uses b = (c-1) mod F */
+  int32_t model;       /* ORC_SSP_LAZY / ORC_ESSP_EAGER / ORC_EXTERNAL */
+  int32_t phased;      /* SSP: 1 = seeded per-worker refresh phase, 0 = none */
+  uint64_t seed;       /* schedule seed */
+  double essp_p;       /* ESSP delay ~ Geometric(essp_p), failures before success */
+  int32_t essp_max_delay;
+  int32_t cap;         /* hot-row step cap C; 0 = off */
+  double eta;          /* step size */
+  double lambda;       /* l2 penalty, per observation */
+  int32_t keep_all;    /* 1 = keep every version (unbounded history) */
+} orc_config;
+
+typedef struct orc_state orc_state;
+
+/* Input arrays are borrowed, not copied, and must outlive the state.
+ * Returns NULL on invalid arguments or allocation failure. */
+orc_state* orc_create(const orc_config* cfg, int64_t n_obs, const int32_t* i, const int32_t* j,
+                      const float* D, const uint8_t* minibatch, const int32_t* user_worker,
+                      const float* L0, const float* R0);
+void orc_destroy(orc_state* st);
+
+/* Run one clock.  v_ext (P entries) is read only for ORC_EXTERNAL.
+ * Returns 0, or -1 on a staleness-bound violation (state unchanged). */
+int orc_clock(orc_state* st, const int32_t* v_ext);
+
+/* Completed clocks (= newest version). */
+int32_t orc_version(const orc_state* st);
+
+/* Read versions used by the last clock, P entries.  Returns -1 before clock 1. */
+int orc_schedule(const orc_state* st, int32_t* v_out);
+
+/* Copy table version `version` ((N+M)*K doubles).  Returns -1 if not held. */
+int orc_table(const orc_state* st, int32_t version, double* out);
+
+/* Objective at `version` over ALL observed entries:
+ * sq = sum e^2 (Sec. 5 squared loss), pen = sum [e^2 + lambda(|L_i|^2+|R_j|^2)]. */
+int orc_objective(const orc_state* st, int32_t version, double* sq, double* pen);
+
+/* The schedule rule alone, for clock c, given the previous read versions.
+ * Used by the schedule tests; orc_clock calls the same function. */
+int orc_schedule_rule(const orc_config* cfg, int32_t c, const int32_t* v_prev, int32_t* v_out);
+
+/* The counter generator (SplitMix64) draw `index` of `stream` under `seed`. */
+uint64_t orc_ctr_u64(uint64_t seed, uint64_t stream, uint64_t index);
+
+#ifdef __cplusplus
+}
+#endif
+#endif
