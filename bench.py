@@ -1,0 +1,430 @@
+"""Benchmark: stale-synchronous MF-SGD clocks on GB300 (ratings per second).
+
+One step = one whole clock of the hot path (read-version schedule, Clock()
+copy of the item rows, fused SGD gather/residual/update/merge) over one
+minibatch of the synthetic Netflix-shaped workload (480k x 18k, 100M
+entries, rank 100, 32 workers, SSP s=3, 1/20 of the data per clock).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload mid]
+    python bench.py --impl reference ...   # the fp64 CPU oracle, same metric
+
+Prints one JSON line.  With N > 1 (torchrun) every rank runs an independent
+replica of the workload on its own GPU: the method has no cross-GPU step.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "SGD ratings/sec per clock on 1 GB300; achieved HBM GB/s vs peak"
+UNIT = "ratings/s"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi SM clock / throttle-reason samples while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.rows = []
+        self.proc = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append((time.time(), line.strip()))
+
+    def mark(self, which):
+        setattr(self, which, time.time())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        rows = [r for t, r in self.rows if self.t0 is None or (self.t0 - 0.1 <= t <= (self.t1 or t) + 0.1)]
+        if not rows:
+            rows = [r for _, r in self.rows]
+        for r in rows:
+            f = [x.strip() for x in r.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for n, val in zip(names, f[4:8]):
+                if val.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def _barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def _max_over_ranks(world, x: float) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _sum_over_ranks(world, x: float) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t)
+    return float(t.item())
+
+
+class FloorModel:
+    """Compulsory HBM bytes of the SGD kernels of one clock (minibatch b, read
+    versions v): 12 B per entry (i, j, D); the merge of every user row (read
+    version c-1, write version c); each user row read at a stale version
+    (v != c-1) by a user with entries; each distinct (item, stale version)
+    row read.  Item rows of version c stay in L2 while deltas fold in."""
+
+    def __init__(self, w, data, wp, mb):
+        self.w = w
+        P, M = w.P, w.n_items
+        self.n = np.zeros(w.F, np.int64)
+        self.users_of = np.zeros((w.F, P), np.int64)
+        self.items_of = []
+        for b in range(w.F):
+            idx = np.flatnonzero(mb == b)
+            ui, jj = data.i[idx], data.j[idx]
+            self.n[b] = idx.size
+            has = np.zeros(w.n_users, bool)
+            has[ui] = True
+            self.users_of[b] = np.bincount(wp[has], minlength=P)
+            m = np.zeros((P, M), bool)
+            m[wp[ui], jj] = True
+            self.items_of.append(m)
+
+    def bytes(self, c, v):
+        w = self.w
+        b = (c - 1) % w.F
+        stale = v != (c - 1)
+        users = int(self.users_of[b][stale].sum())
+        items = 0
+        for ver in np.unique(v[stale]):
+            items += int(np.count_nonzero(self.items_of[b][v == ver].any(axis=0)))
+        return 12 * int(self.n[b]) + 8 * w.K * w.n_users + 4 * w.K * (users + items), int(self.n[b])
+
+
+def run_gpu(args, w):
+    import torch
+
+    from paper_1410_8043_gb300 import esspt
+
+    world, rank, local = _dist()
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    t0 = time.time()
+    data = w.make_data()
+    wp, mb = w.partition()
+    gen_s = time.time() - t0
+    stream = torch.cuda.Stream(dev)
+    with torch.cuda.stream(stream):
+        t = esspt.Table.for_workload(w, data, (wp, mb), device=dev, stream=stream)
+    x0 = torch.as_tensor(np.concatenate([data.L0, data.R0]), device=dev)
+    model = FloorModel(w, data, wp, mb)
+
+    K, W = args.steps, args.warmup
+    # Accounting pass (untimed): read versions of every clock -> floor bytes.
+    floors, counts = [], []
+    for c in range(1, W + K + 1):
+        v, clk = t.read_schedule()
+        assert clk == c
+        if c > W:
+            fb, n = model.bytes(c, v)
+            floors.append(fb)
+            counts.append(n)
+        t.mf_sgd_clock(w.eta, w.lam, w.cap)
+    t.poll()
+    sq0, pen0 = None, None
+
+    # Timed run from version 0 again.
+    t.table_init(x0)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    for a, b_ in ev:  # create the events on the stream
+        a.record(stream)
+        b_.record(stream)
+    for _ in range(W):
+        t.mf_sgd_clock(w.eta, w.lam, w.cap)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    _barrier(world)
+    torch.cuda.synchronize(dev)
+    sampler.mark("t0")
+    start.record(stream)
+    for k in range(K):
+        t.set_profile_events(ev[k][0], ev[k][1])
+        t.mf_sgd_clock(w.eta, w.lam, w.cap)
+    stop.record(stream)
+    torch.cuda.synchronize(dev)
+    sampler.mark("t1")
+    _barrier(world)
+    t.set_profile_events(None, None)
+    clocks = sampler.stop()
+    t.poll()
+    ms = start.elapsed_time(stop)
+    kern_ms = [a.elapsed_time(b_) for a, b_ in ev]
+    ms_max = _max_over_ranks(world, ms)
+    ratings = float(sum(counts))
+    total_ratings = _sum_over_ranks(world, ratings)
+    value = total_ratings / (ms_max / 1e3)
+    c_final = t.clock_index - 1
+    sq, pen = t.mf_objective(c_final, w.lam)
+
+    # End to end through the public API: each step copies its minibatch from
+    # pinned host memory and reads the clock's squared loss back.
+    t.table_init(x0)
+    host_mb = [t.mf_export_minibatch(b) for b in range(w.F)]
+    loss_d = torch.zeros(K, dtype=torch.float64, device=dev)
+    loss_h = torch.empty(K, dtype=torch.float64, pin_memory=True)
+    for _ in range(W):
+        t.mf_sgd_clock(w.eta, w.lam, w.cap)
+    h2d = d2h = 0
+    torch.cuda.synchronize(dev)
+    _barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    wall0 = time.time()
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for k in range(K):
+            c = W + 1 + k
+            b = (c - 1) % w.F
+            u, j, D, uoff = host_mb[b]
+            t.mf_stage_minibatch(b, u, j, D, uoff)
+            h2d += 4 * (u.numel() + j.numel() + D.numel() + uoff.numel())
+            t.mf_sgd_clock(w.eta, w.lam, w.cap, sq_loss=loss_d[k:k + 1])
+            loss_h[k:k + 1].copy_(loss_d[k:k + 1], non_blocking=True)
+            d2h += 8
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    wall = time.time() - wall0
+    _barrier(world)
+    e2e_ms = max(e0.elapsed_time(e1), wall * 1e3)
+    e2e_ms = _max_over_ranks(world, e2e_ms)
+    e2e_value = total_ratings / (e2e_ms / 1e3)
+    t.poll()
+
+    kern_avg_s = statistics.mean(kern_ms) / 1e3
+    floor_avg = statistics.mean(floors)
+    peak, peak_kind = _peaks()
+    achieved = floor_avg / kern_avg_s / 1e9
+    n_avg = ratings / K
+    B_model = 12 + 16 * w.K + 8 * w.K * (w.n_users + w.n_items) / n_avg
+    out = {
+        "metric": METRIC,
+        "value": value,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": ms_max / K,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic (seeded counter generator; Netflix-shaped, no real records)",
+        "config": {
+            "workload": f"{w.name}: {w.n_users}x{w.n_items}, {w.n_obs} entries, rank {w.K}, P={w.P}, "
+                        f"F={w.F}, {w.model.upper()} s={w.s}, eta={w.eta}, lambda={w.lam}, cap={w.cap}",
+            "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
+            "l2": "inputs larger than L2 (version ring %.2f GB, entries %.2f GB; ~%.0f MB streamed per clock)"
+                  % ((w.s + 2) * (w.n_users + w.n_items) * w.K * 4 / 1e9, w.n_obs * 12 / 1e9, floor_avg / 1e6),
+            "ratings_per_clock": n_avg,
+        },
+        "roofline": {
+            "bound": "hbm",
+            "kernel": "sgd_users_kernel (+ sgd_chunks_kernel when present)",
+            "achieved": achieved,
+            "peak": peak,
+            "peak_kind": peak_kind,
+            "unit": "GB/s",
+            "frac": achieved / peak,
+            "traffic": None,
+            "algorithmic_bytes_per_launch": floor_avg,
+            "kernel_ms": statistics.mean(kern_ms),
+            "modelled_bytes_per_rating": B_model,
+            "modelled_GBps": n_avg * B_model / kern_avg_s / 1e9,
+        },
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d // K, "d2h_bytes_per_step": d2h // K},
+        "gpu_launches": K * (3 if t.n_users else 2),
+        "clocks": clocks,
+        "objective": {"clock": c_final, "sq_loss": sq, "penalised": pen},
+        "setup_s": {"generate": gen_s},
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(w, data, (wp, mb), clocks=args.cpu_clocks)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    t.close()
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+def cpu_baseline(w, data, partition, clocks=2):
+    """The fp64 oracle, as it stands, on the first `clocks` clocks of the same
+    workload (single host thread)."""
+    from oracle import Oracle
+
+    o = Oracle.from_workload(w, data, partition)
+    wp, mb = partition
+    n = 0
+    t0 = time.time()
+    for c in range(1, clocks + 1):
+        o.clock()
+        n += int(np.count_nonzero(mb == (c - 1) % w.F))
+    dt = time.time() - t0
+    return {"value": n / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"first {clocks} clocks of {w.name} ({n} entries, full table), fp64, 1 thread",
+            "seconds": dt}
+
+
+def run_reference(args, w):
+    """The oracle as the reference arm: each step is one oracle clock over a
+    bounded sample of the workload (the entries of the first 2% of users,
+    all items, same rank / workers / staleness / step size)."""
+    world, rank, _ = _dist()
+    if rank != 0:
+        return
+    from gen.synth import MFData
+    from oracle import Oracle, OracleConfig
+
+    data = w.make_data()
+    wp, mb = w.partition()
+    n_sub = max(1, w.n_users // 50)
+    keep = data.i < n_sub
+    sub = MFData(n_sub, w.n_items, w.K, data.i[keep], data.j[keep], data.D[keep], data.L0[:n_sub], data.R0)
+    cfg = OracleConfig.from_workload(w, n_users=n_sub)
+    o = Oracle(cfg, sub.i, sub.j, sub.D, mb[keep], wp[:n_sub], sub.L0, sub.R0)
+    mbk = mb[keep]
+    for _ in range(args.warmup):
+        o.clock()
+    n = 0
+    t0 = time.time()
+    for _ in range(args.steps):
+        c = o.version + 1
+        o.clock()
+        n += int(np.count_nonzero(mbk == (c - 1) % w.F))
+    dt = time.time() - t0
+    sample = (f"{w.name} restricted to users [0, {n_sub}) and their {int(keep.sum())} entries, all {w.n_items} "
+              f"items, one oracle clock per step, fp64, 1 thread")
+    out = {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": n / dt,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": dt * 1e3 / args.steps,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": f"{w.name} (bounded sample, see cpu_baseline.sample)"},
+        "cpu_baseline": {"value": n / dt, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": n / dt, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="esspt", choices=["esspt", "reference"])
+    ap.add_argument("--workload", default="mid")
+    ap.add_argument("--cpu-clocks", type=int, default=2)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+    from gen import workload
+
+    w = workload(args.workload)
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_gpu(args, w)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,69 @@
+// Small inline-PTX helpers: vector loads/stores with L2 eviction hints and
+// vector fp32 reductions into global memory (sm_90 and later).
+#pragma once
+
+#include <stdint.h>
+
+namespace esspt {
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// Streaming load: skip L1, mark the L2 lines for early eviction.
+__device__ __forceinline__ float4 ld_stream(const float4* p, uint64_t pol) {
+  float4 r;
+  asm volatile("ld.global.L1::no_allocate.L2::cache_hint.v4.f32 {%0,%1,%2,%3}, [%4], %5;"
+               : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w)
+               : "l"(p), "l"(pol));
+  return r;
+}
+
+// Load that keeps the line in L2 (hot, reused rows).
+__device__ __forceinline__ float4 ld_keep(const float4* p, uint64_t pol) {
+  float4 r;
+  asm volatile("ld.global.L2::cache_hint.v4.f32 {%0,%1,%2,%3}, [%4], %5;"
+               : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w)
+               : "l"(p), "l"(pol));
+  return r;
+}
+
+__device__ __forceinline__ void st_stream(float4* p, float4 v, uint64_t pol) {
+  asm volatile("st.global.L1::no_allocate.L2::cache_hint.v4.f32 [%0], {%1,%2,%3,%4}, %5;"
+               :
+               : "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "l"(pol)
+               : "memory");
+}
+
+// out[0..3] += v, performed at L2 (no return value).
+__device__ __forceinline__ void red_add_v4(float4* p, float4 v) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1,%2,%3,%4};"
+               :
+               : "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
+
+// SplitMix64 (Steele, Lea and Flood, OOPSLA 2014): output n of the sequence
+// whose state starts at s0 is mix64(s0 + n * 0x9E3779B97F4A7C15).
+__host__ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Draw `index` of stream `stream` under `seed`: output index+1 of SplitMix64
+// started at state mix64(seed) ^ mix64(stream).
+__host__ __device__ __forceinline__ uint64_t ctr_u64(uint64_t seed, uint64_t stream, uint64_t index) {
+  const uint64_t s0 = mix64(seed) ^ mix64(stream);
+  return mix64(s0 + (index + 1ull) * 0x9E3779B97F4A7C15ull);
+}
+
+}  // namespace esspt
