@@ -37,7 +37,12 @@ class Workload:
     clocks: int
     eta: float
     lam: float
-    cap: int  # hot-row step cap C (0 = off), see the oracle's header
+    # Hot-row step cap C (0 = off): a row with n > C entries in a clock has
+    # its summed update scaled by C/n.  Summed minibatch updates at the
+    # workloads' step size are unstable on Zipf-popular items without it; C =
+    # 20 keeps eta*C*|L|^2 well inside the stability range of gradient
+    # descent with s clocks of delay (about 2 sin(pi / (2(2s+1)))).
+    cap: int
     data: dict = field(default_factory=dict)
     data_seed: int = DATA_SEED
     sched_seed: int = SCHED_SEED
@@ -87,15 +92,15 @@ WORKLOADS = {
     ),
     "mid": Workload(
         "mid", 480_000, 18_000, 100_000_000, K=100, P=32, F=20, s=3, model="ssp",
-        clocks=40, eta=0.005, lam=0.05, cap=190, data=_MID_DATA,
+        clocks=40, eta=0.005, lam=0.05, cap=20, data=_MID_DATA,
     ),
     "mid_essp": Workload(
         "mid_essp", 480_000, 18_000, 100_000_000, K=100, P=32, F=20, s=3, model="essp",
-        clocks=40, eta=0.005, lam=0.05, cap=190, data=_MID_DATA,
+        clocks=40, eta=0.005, lam=0.05, cap=20, data=_MID_DATA,
     ),
     "large": Workload(
         "large", 10_000_000, 1_000_000, 2_000_000_000, K=64, P=128, F=50, s=4,
-        model="ssp", clocks=20, eta=0.005, lam=0.05, cap=190,
+        model="ssp", clocks=20, eta=0.005, lam=0.05, cap=20,
         data=dict(user_dist="zipf", user_a=1.1, item_dist="zipf", item_a=1.1,
                   truth_rank=32, truth_var=32 ** -0.5, noise_var=0.5),
     ),

@@ -215,8 +215,9 @@ esspt_status esspt_mf_stage_minibatch(esspt_ctx* ctx, int32_t b, const int32_t* 
 
 /* Profiling hook: when `before` and `after` (cudaEvent_t) are non-NULL,
  * every following esspt_mf_sgd_clock() records `before` on the stream just
- * before its SGD kernels and `after` just after them (the Clock() copy of
- * the item rows and the schedule are outside).  NULL, NULL turns it off. */
+ * before its SGD kernels (gather, residual, user-row merge) and `after` just
+ * after them; the item-row Clock() merge and the next clock's schedule come
+ * after `after`.  NULL, NULL turns it off. */
 esspt_status esspt_set_profile_events(esspt_ctx* ctx, void* before, void* after);
 
 #ifdef __cplusplus

@@ -28,10 +28,10 @@ struct esspt_ctx {
   int64_t n_users = 0, n_items = 0, n_obs = 0;
   int32_t F = 0;
   int32_t *rec_u = nullptr, *rec_j = nullptr, *uoff = nullptr, *item_cnt = nullptr, *worker = nullptr;
-  float* rec_D = nullptr;
-  int32_t *chunk_user = nullptr, *chunk_begin = nullptr, *chunk_end = nullptr;
-  int64_t *mb_base_d = nullptr, *chunk_base_d = nullptr;
-  std::vector<int64_t> mb_base, chunk_base;
+  int32_t* item_rep = nullptr;
+  float *rec_D = nullptr, *dR = nullptr, *dL = nullptr;
+  int4 *chunk = nullptr, *heavy = nullptr;
+  std::vector<int64_t> mb_base, chunk_base, heavy_base;
   cudaEvent_t ev_before = nullptr, ev_after = nullptr;
 };
 
@@ -157,25 +157,41 @@ bool is_host_ptr(const void* p) {
 }
 
 struct MfCarve {
-  size_t rec_u, rec_j, rec_D, uoff, mb_base, item_cnt, worker, cu, cb, ce, chunk_base, total;
-  int64_t max_chunks;
+  size_t rec_u, rec_j, rec_D, uoff, mb_base, item_cnt, item_rep, dR, worker, chunk, chunk_base, heavy, heavy_base, dL,
+      total;
+  int64_t max_chunks, max_heavy, dR_rows, dL_rows;
 };
 
-MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F) {
+// Persistent MF workspace: entries laid out by (minibatch, user), per-minibatch
+// user offsets and item counts, item replica rows, heavy-user lists and the
+// zero-initialised delta replicas dR (items) and dL (heavy users).
+MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int32_t K) {
   MfCarve k{};
   k.max_chunks = layout_max_chunks(n_obs, F);
+  k.max_heavy = layout_max_heavy(n_obs, F);
+  k.dR_rows = layout_max_item_reps(n_obs, n_items);
+  k.dL_rows = n_users + layout_max_user_reps(n_obs);
   size_t o = 0;
-  k.rec_u = o; o += align256(sizeof(int32_t) * n_obs);
-  k.rec_j = o; o += align256(sizeof(int32_t) * n_obs);
-  k.rec_D = o; o += align256(sizeof(float) * n_obs);
-  k.uoff = o; o += align256(sizeof(int32_t) * (size_t)F * (n_users + 1));
-  k.mb_base = o; o += align256(sizeof(int64_t) * (F + 1));
-  k.item_cnt = o; o += align256(sizeof(int32_t) * (size_t)F * n_items);
-  k.worker = o; o += align256(sizeof(int32_t) * n_users);
-  k.cu = o; o += align256(sizeof(int32_t) * k.max_chunks);
-  k.cb = o; o += align256(sizeof(int32_t) * k.max_chunks);
-  k.ce = o; o += align256(sizeof(int32_t) * k.max_chunks);
-  k.chunk_base = o; o += align256(sizeof(int64_t) * (F + 1));
+  auto take = [&o](size_t bytes) {
+    const size_t at = o;
+    o += align256(bytes);
+    return at;
+  };
+  // 16 bytes of slack past the entry arrays for vector-aligned staging.
+  k.rec_u = take(sizeof(int32_t) * (n_obs + 4));
+  k.rec_j = take(sizeof(int32_t) * (n_obs + 4));
+  k.rec_D = take(sizeof(float) * (n_obs + 4));
+  k.uoff = take(sizeof(int32_t) * (size_t)F * (n_users + 1));
+  k.mb_base = take(sizeof(int64_t) * (F + 1));
+  k.item_cnt = take(sizeof(int32_t) * (size_t)F * n_items);
+  k.item_rep = take(sizeof(int32_t) * (n_items + 1));
+  k.dR = take(sizeof(float) * (size_t)k.dR_rows * K);
+  k.worker = take(sizeof(int32_t) * n_users);
+  k.chunk = take(sizeof(int4) * k.max_chunks);
+  k.chunk_base = take(sizeof(int64_t) * (F + 1));
+  k.heavy = take(sizeof(int4) * k.max_heavy);
+  k.heavy_base = take(sizeof(int64_t) * (F + 1));
+  k.dL = take(sizeof(float) * (size_t)k.dL_rows * K);
   k.total = o;
   return k;
 }
@@ -348,12 +364,12 @@ esspt_status esspt_read_table(esspt_ctx* c, int32_t version, float* out) {
 
 size_t esspt_mf_workspace_bytes(const esspt_ctx* c, int64_t n_obs, int64_t n_users, int32_t F) {
   if (!mf_sizes_ok(c, n_obs, n_users, F)) return 0;
-  return mf_carve(n_obs, n_users, c->n_rows - n_users, F).total;
+  return mf_carve(n_obs, n_users, c->n_rows - n_users, F, c->K).total;
 }
 
 size_t esspt_mf_scratch_bytes(const esspt_ctx* c, int64_t n_obs, int64_t n_users, int32_t F) {
   if (!mf_sizes_ok(c, n_obs, n_users, F)) return 0;
-  return layout_scratch_bytes(n_obs, n_users, F);
+  return layout_scratch_bytes(n_obs, n_users, c->n_rows - n_users, F);
 }
 
 esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j, const float* d_D,
@@ -366,9 +382,10 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   if ((reinterpret_cast<uintptr_t>(d_ws) & 255u) || (reinterpret_cast<uintptr_t>(d_scratch) & 255u))
     return fail(c, ESSPT_EINVAL, "MF buffers must be 256-byte aligned");
   const int64_t n_items = c->n_rows - n_users;
-  const MfCarve k = mf_carve(n_obs, n_users, n_items, F);
+  const MfCarve k = mf_carve(n_obs, n_users, n_items, F, c->K);
   if (bytes < k.total) return fail(c, ESSPT_ENOSPC, "MF workspace too small");
-  if (scratch_bytes < layout_scratch_bytes(n_obs, n_users, F)) return fail(c, ESSPT_ENOSPC, "MF scratch too small");
+  if (scratch_bytes < layout_scratch_bytes(n_obs, n_users, n_items, F))
+    return fail(c, ESSPT_ENOSPC, "MF scratch too small");
   c->mf = false;
   char* w = static_cast<char*>(d_ws);
   LayoutBuild b{};
@@ -388,11 +405,13 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   b.uoff = reinterpret_cast<int32_t*>(w + k.uoff);
   b.mb_base = reinterpret_cast<int64_t*>(w + k.mb_base);
   b.item_cnt = reinterpret_cast<int32_t*>(w + k.item_cnt);
-  b.chunk_user = reinterpret_cast<int32_t*>(w + k.cu);
-  b.chunk_begin = reinterpret_cast<int32_t*>(w + k.cb);
-  b.chunk_end = reinterpret_cast<int32_t*>(w + k.ce);
+  b.item_rep = reinterpret_cast<int32_t*>(w + k.item_rep);
+  b.chunk = reinterpret_cast<int4*>(w + k.chunk);
   b.chunk_base = reinterpret_cast<int64_t*>(w + k.chunk_base);
+  b.heavy = reinterpret_cast<int4*>(w + k.heavy);
+  b.heavy_base = reinterpret_cast<int64_t*>(w + k.heavy_base);
   b.max_chunks = k.max_chunks;
+  b.max_heavy = k.max_heavy;
   b.scratch = d_scratch;
   b.scratch_bytes = scratch_bytes;
   b.status = c->status;
@@ -408,13 +427,21 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   }
   int32_t* worker = reinterpret_cast<int32_t*>(w + k.worker);
   ESSPT_CUDA(c, cudaMemcpyAsync(worker, d_worker, sizeof(int32_t) * n_users, cudaMemcpyDeviceToDevice, c->st));
+  float* dR = reinterpret_cast<float*>(w + k.dR);
+  float* dL = reinterpret_cast<float*>(w + k.dL);
+  ESSPT_CUDA(c, cudaMemsetAsync(dR, 0, sizeof(float) * (size_t)k.dR_rows * c->K, c->st));
+  ESSPT_CUDA(c, cudaMemsetAsync(dL, 0, sizeof(float) * (size_t)k.dL_rows * c->K, c->st));
+  ESSPT_CUDA(c, cudaMemsetAsync(b.rec_u + n_obs, 0, 16, c->st));
+  ESSPT_CUDA(c, cudaMemsetAsync(b.rec_j + n_obs, 0, 16, c->st));
+  ESSPT_CUDA(c, cudaMemsetAsync(b.rec_D + n_obs, 0, 16, c->st));
   ESSPT_CUDA(c, build_layout(b, c->st));
-  std::vector<int64_t> mbb((size_t)F + 1), chb((size_t)F + 1);
+  std::vector<int64_t> mbb((size_t)F + 1), chb((size_t)F + 1), hvb((size_t)F + 1);
   ESSPT_CUDA(c, cudaMemcpyAsync(mbb.data(), b.mb_base, sizeof(int64_t) * (F + 1), cudaMemcpyDeviceToHost, c->st));
   ESSPT_CUDA(c, cudaMemcpyAsync(chb.data(), b.chunk_base, sizeof(int64_t) * (F + 1), cudaMemcpyDeviceToHost, c->st));
+  ESSPT_CUDA(c, cudaMemcpyAsync(hvb.data(), b.heavy_base, sizeof(int64_t) * (F + 1), cudaMemcpyDeviceToHost, c->st));
   ESSPT_CUDA(c, cudaMemcpyAsync(&bits, c->status, sizeof bits, cudaMemcpyDeviceToHost, c->st));
   ESSPT_CUDA(c, cudaStreamSynchronize(c->st));
-  if (chb[F] > k.max_chunks || (bits & kErrInput)) {
+  if (chb[F] > k.max_chunks || hvb[F] > k.max_heavy || (bits & kErrInput)) {
     ESSPT_CUDA(c, cudaMemsetAsync(c->status, 0, sizeof(uint32_t), c->st));
     return fail(c, ESSPT_ECUDA, "internal: chunk list overflow");
   }
@@ -428,13 +455,14 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   c->uoff = b.uoff;
   c->item_cnt = b.item_cnt;
   c->worker = worker;
-  c->chunk_user = b.chunk_user;
-  c->chunk_begin = b.chunk_begin;
-  c->chunk_end = b.chunk_end;
-  c->mb_base_d = b.mb_base;
-  c->chunk_base_d = b.chunk_base;
+  c->item_rep = b.item_rep;
+  c->dR = dR;
+  c->dL = dL;
+  c->chunk = b.chunk;
+  c->heavy = b.heavy;
   c->mb_base = mbb;
   c->chunk_base = chb;
+  c->heavy_base = hvb;
   c->mf = true;
   return ESSPT_OK;
 }
@@ -446,44 +474,72 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   if ((s = need_schedule(c)) != ESSPT_OK) return s;
   if (cap < 0) return fail(c, ESSPT_EINVAL, "cap must be >= 0");
   const int32_t b = (c->clock - 1) % c->F;
+  // Version c is merged from version c-1, or in place when INCs already
+  // initialised it during this clock.
+  const int32_t slot_out = c->clock % c->nslots;
+  const int32_t slot_base = c->acc_ready ? slot_out : (c->clock - 1) % c->nslots;
   SgdArgs a{};
   a.ring = c->ring;
   a.n_rows = c->n_rows;
   a.K = c->K;
   a.n_users = (int32_t)c->n_users;
   a.nslots = c->nslots;
-  a.slot_out = c->clock % c->nslots;
-  if (c->acc_ready) {
-    a.slot_base = a.slot_out;  // INCs already landed in version c: merge in place
-  } else {
-    a.slot_base = (c->clock - 1) % c->nslots;
-    const int64_t r0 = c->n_users * (int64_t)c->K;
-    ESSPT_CUDA(c, launch_copy_rows(slot_ptr(c, c->clock) + r0, slot_ptr(c, c->clock - 1) + r0,
-                                   c->n_items * (int64_t)c->K, c->st));
-  }
+  a.slot_base = slot_base;
+  a.slot_out = slot_out;
+  a.n_b = (int32_t)(c->mb_base[b + 1] - c->mb_base[b]);
   a.v = c->v;
   a.worker = c->worker;
   a.uoff = c->uoff + (int64_t)b * (c->n_users + 1);
   a.rec_j = c->rec_j + c->mb_base[b];
   a.rec_D = c->rec_D + c->mb_base[b];
-  a.item_cnt = c->item_cnt + (int64_t)b * c->n_items;
+  a.item_rep = c->item_rep;
+  a.dR = c->dR;
   a.eta = eta;
   a.lambda = lambda;
   a.cap = cap;
   a.sq_loss = d_sq_loss;
-  if (c->ev_before) ESSPT_CUDA(c, cudaEventRecord(c->ev_before, c->st));
-  ESSPT_CUDA(c, launch_sgd_users(a, c->st));
   const int64_t nch = c->chunk_base[b + 1] - c->chunk_base[b];
+  const int64_t nhv = c->heavy_base[b + 1] - c->heavy_base[b];
+  if (c->ev_before) ESSPT_CUDA(c, cudaEventRecord(c->ev_before, c->st));
   if (nch > 0) {
     ChunkArgs ch{};
     ch.a = a;
-    ch.chunk_user = c->chunk_user + c->chunk_base[b];
-    ch.chunk_begin = c->chunk_begin + c->chunk_base[b];
-    ch.chunk_end = c->chunk_end + c->chunk_base[b];
+    ch.chunk = c->chunk + c->chunk_base[b];
     ch.n_chunks = nch;
+    ch.dL = c->dL;
     ESSPT_CUDA(c, launch_sgd_chunks(ch, c->st));
   }
+  ESSPT_CUDA(c, launch_sgd_users(a, c->st));
+  if (nhv > 0) {
+    HeavyMergeArgs h{};
+    h.ring = c->ring;
+    h.n_rows = c->n_rows;
+    h.K = c->K;
+    h.nslots = c->nslots;
+    h.slot_base = slot_base;
+    h.slot_out = slot_out;
+    h.heavy = c->heavy + c->heavy_base[b];
+    h.n_heavy = nhv;
+    h.dL = c->dL;
+    h.eta = eta;
+    h.cap = cap;
+    ESSPT_CUDA(c, launch_heavy_merge(h, c->st));
+  }
   if (c->ev_after) ESSPT_CUDA(c, cudaEventRecord(c->ev_after, c->st));
+  ItemMergeArgs m{};
+  m.ring = c->ring;
+  m.n_rows = c->n_rows;
+  m.K = c->K;
+  m.n_users = (int32_t)c->n_users;
+  m.n_items = (int32_t)c->n_items;
+  m.slot_base = slot_base;
+  m.slot_out = slot_out;
+  m.item_rep = c->item_rep;
+  m.dR = c->dR;
+  m.item_cnt = c->item_cnt + (int64_t)b * c->n_items;
+  m.eta = eta;
+  m.cap = cap;
+  ESSPT_CUDA(c, launch_item_merge(m, c->st));
   c->acc_ready = true;
   return advance(c);
 }

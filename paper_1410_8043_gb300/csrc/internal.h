@@ -19,9 +19,17 @@ enum : uint32_t {
 constexpr uint64_t kStreamPhase = 101u;
 constexpr uint64_t kStreamDelay = 102u;
 
-// Entries per chunk for users whose clock segment exceeds kHeavy entries.
+// Users with more than kHeavy entries in a minibatch are split in chunks of
+// kChunk entries, processed apart from the per-user kernel.
 constexpr int32_t kHeavy = 96;
 constexpr int32_t kChunk = 64;
+// Replica accumulators: an item gets one delta row per kItemRep entries
+// (largest minibatch count, rounded up to a power of two); a heavy user one
+// per kUserRep chunks.  Replicas spread the fp32 reductions of popular rows
+// over many L2 addresses and keep each partial sum short.
+constexpr int32_t kItemRep = 2048;
+constexpr int32_t kUserRep = 64;
+constexpr int32_t kMaxRep = 512;
 
 struct ScheduleArgs {
   int32_t* v;              // [P] read versions (in: v(c-1), out: v(c))
@@ -31,32 +39,58 @@ struct ScheduleArgs {
   uint64_t seed;
 };
 
-// Fused MF-SGD clock over the users of one minibatch.
+// One clock of MF-SGD over the users of minibatch b.
 struct SgdArgs {
-  float* ring;             // (s+2) * n_rows * K
+  float* ring;              // (s+2) * n_rows * K
   int64_t n_rows;
   int32_t K;
   int32_t n_users;
-  int32_t nslots;          // s + 2
-  int32_t slot_base;       // slot the L rows are merged from (c-1, or c if INCs happened)
-  int32_t slot_out;        // slot of version c
-  const int32_t* v;        // [P] read versions
-  const int32_t* worker;   // [n_users]
-  const int32_t* uoff;     // [n_users+1] entry offsets of minibatch b, relative to its base
-  const int32_t* rec_j;    // item of each entry (minibatch base applied)
-  const float* rec_D;      // value of each entry
-  const int32_t* item_cnt; // [M] entries per item in minibatch b
+  int32_t nslots;           // s + 2
+  int32_t slot_base;        // slot merged from (c-1, or c if INCs already landed there)
+  int32_t slot_out;         // slot of version c
+  int32_t n_b;              // entries of minibatch b
+  const int32_t* v;         // [P] read versions
+  const int32_t* worker;    // [n_users]
+  const int32_t* uoff;      // [n_users+1] entry offsets of minibatch b (relative)
+  const int32_t* rec_j;     // item of each entry of minibatch b
+  const float* rec_D;       // value of each entry of minibatch b
+  const int32_t* item_rep;  // [M+1] first replica row of each item in dR
+  float* dR;                // item delta replicas (all zero between clocks)
   float eta, lambda;
   int32_t cap;
-  double* sq_loss;         // optional
+  double* sq_loss;          // optional
 };
 
+// Chunks of heavy users: x = user, y = begin, z = end (relative), w = replica row in dL.
 struct ChunkArgs {
   SgdArgs a;
-  const int32_t* chunk_user;   // [n_chunks]
-  const int32_t* chunk_begin;  // relative to the minibatch base
-  const int32_t* chunk_end;
+  const int4* chunk;
   int64_t n_chunks;
+  float* dL;                // heavy-user delta replicas (all zero between clocks)
+};
+
+// Merge of heavy user rows: x = user, y = first replica row, z = replicas, w = entries.
+struct HeavyMergeArgs {
+  float* ring;
+  int64_t n_rows;
+  int32_t K, nslots, slot_base, slot_out;
+  const int4* heavy;
+  int64_t n_heavy;
+  float* dL;
+  float eta;
+  int32_t cap;
+};
+
+// Clock() merge of the item rows: R^c_j = R^base_j + eta s_j sum of replicas.
+struct ItemMergeArgs {
+  float* ring;
+  int64_t n_rows;
+  int32_t K, n_users, n_items, slot_base, slot_out;
+  const int32_t* item_rep;
+  float* dR;
+  const int32_t* item_cnt;  // [M] entries per item in minibatch b
+  float eta;
+  int32_t cap;
 };
 
 // Launchers (return the launch error, if any).
@@ -69,6 +103,8 @@ cudaError_t launch_inc(float* slot, int64_t n_rows, int32_t K, const int32_t* id
                        uint32_t* status, cudaStream_t st);
 cudaError_t launch_sgd_users(const SgdArgs& a, cudaStream_t st);
 cudaError_t launch_sgd_chunks(const ChunkArgs& a, cudaStream_t st);
+cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st);
+cudaError_t launch_item_merge(const ItemMergeArgs& a, cudaStream_t st);
 cudaError_t launch_objective(const float* slot, int64_t n_users, int32_t K, const int32_t* rec_u,
                              const int32_t* rec_j, const float* rec_D, int64_t n_obs, float lambda,
                              double* out2, cudaStream_t st);
@@ -89,19 +125,23 @@ struct LayoutBuild {
   int32_t* uoff;        // [F][n_users+1]
   int64_t* mb_base;     // [F+1]
   int32_t* item_cnt;    // [F][n_items]
-  int32_t* chunk_user;  // [max_chunks]
-  int32_t* chunk_begin;
-  int32_t* chunk_end;
+  int32_t* item_rep;    // [n_items+1]
+  int4* chunk;          // [max_chunks]
   int64_t* chunk_base;  // [F+1]
-  int64_t max_chunks;
+  int4* heavy;          // [max_heavy]
+  int64_t* heavy_base;  // [F+1]
+  int64_t max_chunks, max_heavy;
   // scratch
   void* scratch;
   size_t scratch_bytes;
   uint32_t* status;
 };
 
-size_t layout_scratch_bytes(int64_t n_obs, int64_t n_users, int32_t F);
+size_t layout_scratch_bytes(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F);
 int64_t layout_max_chunks(int64_t n_obs, int32_t F);
+int64_t layout_max_heavy(int64_t n_obs, int32_t F);
+int64_t layout_max_item_reps(int64_t n_obs, int64_t n_items);
+int64_t layout_max_user_reps(int64_t n_obs);
 cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st);
 cudaError_t launch_validate(const LayoutBuild& b, cudaStream_t st);
 

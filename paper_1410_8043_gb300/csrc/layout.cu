@@ -2,7 +2,9 @@
 // minibatch and user so that a clock streams one contiguous, user-sorted
 // segment (Sec. 3.1: D_obs partitioned over workers; Sec. 5: a fixed
 // minibatch per Clock()).  The radix sort is stable, so entries of a user
-// keep their input order and every run sees the same layout.
+// keep their input order and every run sees the same layout.  Also builds
+// the chunk and heavy-user lists and the replica rows of popular items and
+// heavy users.
 #include <algorithm>
 
 #include <cub/device/device_radix_sort.cuh>
@@ -15,6 +17,26 @@ namespace esspt {
 namespace {
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+__host__ __device__ inline int32_t next_pow2(int32_t x) {
+  int32_t p = 1;
+  while (p < x) p <<= 1;
+  return p;
+}
+
+// Replicas of a heavy user with nch chunks: one per kUserRep chunks, rounded
+// up to a power of two (never more than nch), at most kMaxRep.
+__host__ __device__ inline int32_t user_reps(int32_t nch) {
+  const int32_t r = next_pow2((nch + kUserRep - 1) / kUserRep);
+  return r < kMaxRep ? r : kMaxRep;
+}
+
+// Replicas of an item whose largest minibatch count is mx, at most kMaxRep.
+__host__ __device__ inline int32_t item_reps(int32_t mx) {
+  const int32_t want = (mx + kItemRep - 1) / kItemRep;
+  const int32_t r = next_pow2(want > 1 ? want : 1);
+  return r < kMaxRep ? r : kMaxRep;
+}
 
 __global__ void validate_kernel(const int32_t* __restrict__ i, const int32_t* __restrict__ j,
                                 const uint8_t* __restrict__ mb, int64_t n_obs, const int32_t* __restrict__ worker,
@@ -54,10 +76,11 @@ __global__ void gather_kernel(const uint32_t* __restrict__ perm, int64_t n_obs, 
   }
 }
 
-// uoff[b][u] = off[b*N+u] - off[b*N] for u in [0, N]; mb_base[b] = off[b*N].
+// uoff[b][u] = off[b*N+u] - off[b*N] for u in [0, N]; mb_base[b] = off[b*N];
+// per (b, u): chunks, heavy flag and extra replica rows.
 __global__ void offsets_kernel(const int64_t* __restrict__ off, int64_t n_users, int32_t F, int32_t* __restrict__ uoff,
                                int64_t* __restrict__ mb_base, const int32_t* __restrict__ cnt,
-                               int32_t* __restrict__ nchunks) {
+                               int32_t* __restrict__ nch, int32_t* __restrict__ hflag, int32_t* __restrict__ hextra) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t total = (int64_t)F * (n_users + 1);
   for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < total; x += stride) {
@@ -67,36 +90,64 @@ __global__ void offsets_kernel(const int64_t* __restrict__ off, int64_t n_users,
     if (u == 0) mb_base[b] = base;
     if (u < n_users) {
       const int32_t n = cnt[b * n_users + u];
-      nchunks[b * n_users + u] = n > kHeavy ? (n + kChunk - 1) / kChunk : 0;
+      const int32_t c = n > kHeavy ? (n + kChunk - 1) / kChunk : 0;
+      nch[b * n_users + u] = c;
+      hflag[b * n_users + u] = c > 0 ? 1 : 0;
+      hextra[b * n_users + u] = c > 0 ? user_reps(c) - 1 : 0;
     }
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) mb_base[F] = off[(int64_t)F * n_users];
 }
 
-__global__ void chunks_kernel(const int64_t* __restrict__ choff, const int32_t* __restrict__ nchunks,
-                              const int32_t* __restrict__ uoff, int64_t n_users, int32_t F,
-                              int32_t* __restrict__ cu, int32_t* __restrict__ cb, int32_t* __restrict__ ce,
-                              int64_t* __restrict__ chunk_base, int64_t max_chunks, uint32_t* status) {
+// Chunk descriptors (user, begin, end, replica row) and heavy-user
+// descriptors (user, first extra replica row, replicas, entries).  Replica 0
+// of heavy user u is row u of dL; replicas 1.. are rows n_users + hext[...].
+__global__ void heavy_kernel(const int64_t* __restrict__ choff, const int32_t* __restrict__ nch,
+                             const int64_t* __restrict__ hoff, const int64_t* __restrict__ hext,
+                             const int32_t* __restrict__ uoff, int64_t n_users, int32_t F, int4* __restrict__ chunk,
+                             int64_t* __restrict__ chunk_base, int64_t max_chunks, int4* __restrict__ heavy,
+                             int64_t* __restrict__ heavy_base, int64_t max_heavy, int64_t max_user_reps,
+                             uint32_t* status) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t total = (int64_t)F * n_users;
   for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < total; x += stride) {
-    const int32_t nc = nchunks[x];
+    const int32_t nc = nch[x];
     if (nc == 0) continue;
     const int64_t b = x / n_users, u = x % n_users;
     const int32_t beg = uoff[b * (n_users + 1) + u], end = uoff[b * (n_users + 1) + u + 1];
+    const int32_t reps = user_reps(nc);
+    const int64_t extra0 = n_users + hext[x];
+    // The bounds below hold by construction; the checks keep every store in range.
+    if (hoff[x] >= max_heavy || choff[x] + nc > max_chunks || hext[x] + reps - 1 > max_user_reps) {
+      atomicOr(status, kErrInput);
+      continue;
+    }
+    heavy[hoff[x]] = make_int4((int32_t)u, (int32_t)extra0, reps, end - beg);
     for (int32_t t = 0; t < nc; ++t) {
-      const int64_t k = choff[x] + t;
-      if (k >= max_chunks) {  // cannot happen: sum of ceil(n/kChunk) over n > kHeavy is < 2 n_obs / kChunk
-        atomicOr(status, kErrInput);
-        break;
-      }
-      cu[k] = (int32_t)u;
-      cb[k] = beg + t * kChunk;
-      ce[k] = min(end, beg + (t + 1) * kChunk);
+      const int32_t r = t & (reps - 1);
+      const int32_t dst = r == 0 ? (int32_t)u : (int32_t)(extra0 + r - 1);
+      chunk[choff[x] + t] = make_int4((int32_t)u, beg + t * kChunk, min(end, beg + (t + 1) * kChunk), dst);
     }
   }
-  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b <= F; b += stride)
+  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b <= F; b += stride) {
     chunk_base[b] = choff[b * n_users];
+    heavy_base[b] = hoff[b * n_users];
+  }
+}
+
+// Replica count of every item from its largest minibatch count.
+__global__ void item_reps_kernel(const int32_t* __restrict__ item_cnt, int64_t n_items, int32_t F,
+                                 int32_t* __restrict__ reps) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j <= n_items; j += stride) {
+    if (j == n_items) {
+      reps[j] = 0;
+      continue;
+    }
+    int32_t mx = 0;
+    for (int32_t b = 0; b < F; ++b) mx = max(mx, item_cnt[(int64_t)b * n_items + j]);
+    reps[j] = item_reps(mx);
+  }
 }
 
 int blocks_for(int64_t n) {
@@ -107,32 +158,41 @@ int blocks_for(int64_t n) {
 }
 
 struct ScratchPlan {
-  size_t key_in, key_out, val_in, val_out, cnt, off, nchunks, choff, cub, total;
+  size_t key_in, key_out, val_in, val_out, cnt, off, nch, choff, hflag, hoff, hextra, hext, ireps, cub, total;
   size_t cub_bytes;
 };
 
-ScratchPlan plan(int64_t n_obs, int64_t n_users, int32_t F) {
+ScratchPlan plan(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F) {
   ScratchPlan p{};
   const int64_t keys = (int64_t)F * n_users;
   size_t sort_bytes = 0, scan_bytes = 0, scan2_bytes = 0;
   cub::DeviceRadixSort::SortPairs(nullptr, sort_bytes, (const uint32_t*)nullptr, (uint32_t*)nullptr,
                                   (const uint32_t*)nullptr, (uint32_t*)nullptr, (int)std::max<int64_t>(n_obs, 1), 0,
                                   32);
-  cub::DeviceScan::ExclusiveSum(nullptr, scan_bytes, (const int32_t*)nullptr, (int64_t*)nullptr,
-                                (int)(keys + 1));
-  cub::DeviceScan::ExclusiveSum(nullptr, scan2_bytes, (const int32_t*)nullptr, (int64_t*)nullptr,
-                                (int)(keys + 1));
+  cub::DeviceScan::ExclusiveSum(nullptr, scan_bytes, (const int32_t*)nullptr, (int64_t*)nullptr, (int)(keys + 1));
+  cub::DeviceScan::ExclusiveSum(nullptr, scan2_bytes, (const int32_t*)nullptr, (int32_t*)nullptr,
+                                (int)(n_items + 1));
   p.cub_bytes = std::max(sort_bytes, std::max(scan_bytes, scan2_bytes));
   size_t o = 0;
-  p.key_in = o; o += align256(sizeof(uint32_t) * n_obs);
-  p.key_out = o; o += align256(sizeof(uint32_t) * n_obs);
-  p.val_in = o; o += align256(sizeof(uint32_t) * n_obs);
-  p.val_out = o; o += align256(sizeof(uint32_t) * n_obs);
-  p.cnt = o; o += align256(sizeof(int32_t) * (keys + 1));
-  p.off = o; o += align256(sizeof(int64_t) * (keys + 1));
-  p.nchunks = o; o += align256(sizeof(int32_t) * (keys + 1));
-  p.choff = o; o += align256(sizeof(int64_t) * (keys + 1));
-  p.cub = o; o += align256(p.cub_bytes);
+  auto take = [&o](size_t bytes) {
+    const size_t at = o;
+    o += align256(bytes);
+    return at;
+  };
+  p.key_in = take(sizeof(uint32_t) * n_obs);
+  p.key_out = take(sizeof(uint32_t) * n_obs);
+  p.val_in = take(sizeof(uint32_t) * n_obs);
+  p.val_out = take(sizeof(uint32_t) * n_obs);
+  p.cnt = take(sizeof(int32_t) * (keys + 1));
+  p.off = take(sizeof(int64_t) * (keys + 1));
+  p.nch = take(sizeof(int32_t) * (keys + 1));
+  p.choff = take(sizeof(int64_t) * (keys + 1));
+  p.hflag = take(sizeof(int32_t) * (keys + 1));
+  p.hoff = take(sizeof(int64_t) * (keys + 1));
+  p.hextra = take(sizeof(int32_t) * (keys + 1));
+  p.hext = take(sizeof(int64_t) * (keys + 1));
+  p.ireps = take(sizeof(int32_t) * (n_items + 1));
+  p.cub = take(p.cub_bytes);
   p.total = o;
   return p;
 }
@@ -145,15 +205,23 @@ int bits_for(uint64_t max_key) {
 
 }  // namespace
 
-size_t layout_scratch_bytes(int64_t n_obs, int64_t n_users, int32_t F) { return plan(n_obs, n_users, F).total; }
-
-int64_t layout_max_chunks(int64_t n_obs, int32_t F) {
-  // A heavy segment has n > kHeavy >= kChunk entries and ceil(n/kChunk) <= 2n/kChunk chunks.
-  return 2 * n_obs / kChunk + F + 1;
+size_t layout_scratch_bytes(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F) {
+  return plan(n_obs, n_users, n_items, F).total;
 }
 
+// A heavy segment has n > kHeavy >= kChunk entries and ceil(n/kChunk) < 2n/kChunk chunks.
+int64_t layout_max_chunks(int64_t n_obs, int32_t F) { return 2 * n_obs / kChunk + F + 1; }
+
+int64_t layout_max_heavy(int64_t n_obs, int32_t F) { return n_obs / (kHeavy + 1) + F + 1; }
+
+// sum over items of replicas: n_items + sum (reps - 1), and reps - 1 < 3 mx / (2 kItemRep).
+int64_t layout_max_item_reps(int64_t n_obs, int64_t n_items) { return n_items + 3 * n_obs / (2 * kItemRep) + 2; }
+
+// Extra replica rows of heavy users: reps - 1 < 3 nch / (2 kUserRep), sum nch < 2 n_obs / kChunk.
+int64_t layout_max_user_reps(int64_t n_obs) { return 3 * n_obs / (kChunk * kUserRep) + 2; }
+
 cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st) {
-  const ScratchPlan p = plan(b.n_obs, b.n_users, b.F);
+  const ScratchPlan p = plan(b.n_obs, b.n_users, b.n_items, b.F);
   if (b.scratch_bytes < p.total) return cudaErrorInvalidValue;
   char* s = static_cast<char*>(b.scratch);
   uint32_t* key_in = reinterpret_cast<uint32_t*>(s + p.key_in);
@@ -162,14 +230,19 @@ cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st) {
   uint32_t* val_out = reinterpret_cast<uint32_t*>(s + p.val_out);
   int32_t* cnt = reinterpret_cast<int32_t*>(s + p.cnt);
   int64_t* off = reinterpret_cast<int64_t*>(s + p.off);
-  int32_t* nch = reinterpret_cast<int32_t*>(s + p.nchunks);
+  int32_t* nch = reinterpret_cast<int32_t*>(s + p.nch);
   int64_t* choff = reinterpret_cast<int64_t*>(s + p.choff);
+  int32_t* hflag = reinterpret_cast<int32_t*>(s + p.hflag);
+  int64_t* hoff = reinterpret_cast<int64_t*>(s + p.hoff);
+  int32_t* hextra = reinterpret_cast<int32_t*>(s + p.hextra);
+  int64_t* hext = reinterpret_cast<int64_t*>(s + p.hext);
+  int32_t* ireps = reinterpret_cast<int32_t*>(s + p.ireps);
   void* cub_tmp = s + p.cub;
   const int64_t keys = (int64_t)b.F * b.n_users;
   cudaError_t e;
 
-  if ((e = cudaMemsetAsync(cnt, 0, sizeof(int32_t) * (keys + 1), st)) != cudaSuccess) return e;
-  if ((e = cudaMemsetAsync(nch, 0, sizeof(int32_t) * (keys + 1), st)) != cudaSuccess) return e;
+  for (void* z : {(void*)cnt, (void*)nch, (void*)hflag, (void*)hextra})
+    if ((e = cudaMemsetAsync(z, 0, sizeof(int32_t) * (keys + 1), st)) != cudaSuccess) return e;
   if ((e = cudaMemsetAsync(b.item_cnt, 0, sizeof(int32_t) * b.F * b.n_items, st)) != cudaSuccess) return e;
   keys_kernel<<<blocks_for(b.n_obs), 256, 0, st>>>(b.i, b.j, b.mb, b.n_obs, b.n_users, b.n_items, key_in, val_in, cnt,
                                                   b.item_cnt);
@@ -185,13 +258,22 @@ cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st) {
   size_t tb = p.cub_bytes;
   if ((e = cub::DeviceScan::ExclusiveSum(cub_tmp, tb, cnt, off, (int)(keys + 1), st)) != cudaSuccess) return e;
   offsets_kernel<<<blocks_for((int64_t)b.F * (b.n_users + 1)), 256, 0, st>>>(off, b.n_users, b.F, b.uoff, b.mb_base,
-                                                                            cnt, nch);
+                                                                            cnt, nch, hflag, hextra);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   tb = p.cub_bytes;
   if ((e = cub::DeviceScan::ExclusiveSum(cub_tmp, tb, nch, choff, (int)(keys + 1), st)) != cudaSuccess) return e;
-  chunks_kernel<<<blocks_for(keys + 1), 256, 0, st>>>(choff, nch, b.uoff, b.n_users, b.F, b.chunk_user, b.chunk_begin,
-                                                      b.chunk_end, b.chunk_base, b.max_chunks, b.status);
-  return cudaGetLastError();
+  tb = p.cub_bytes;
+  if ((e = cub::DeviceScan::ExclusiveSum(cub_tmp, tb, hflag, hoff, (int)(keys + 1), st)) != cudaSuccess) return e;
+  tb = p.cub_bytes;
+  if ((e = cub::DeviceScan::ExclusiveSum(cub_tmp, tb, hextra, hext, (int)(keys + 1), st)) != cudaSuccess) return e;
+  heavy_kernel<<<blocks_for(keys + 1), 256, 0, st>>>(choff, nch, hoff, hext, b.uoff, b.n_users, b.F, b.chunk,
+                                                     b.chunk_base, b.max_chunks, b.heavy, b.heavy_base, b.max_heavy,
+                                                     layout_max_user_reps(b.n_obs), b.status);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  item_reps_kernel<<<blocks_for(b.n_items + 1), 256, 0, st>>>(b.item_cnt, b.n_items, b.F, ireps);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  tb = p.cub_bytes;
+  return cub::DeviceScan::ExclusiveSum(cub_tmp, tb, ireps, b.item_rep, (int)(b.n_items + 1), st);
 }
 
 cudaError_t launch_validate(const LayoutBuild& b, cudaStream_t st) {

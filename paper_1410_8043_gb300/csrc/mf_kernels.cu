@@ -1,7 +1,14 @@
 // Matrix-factorisation SGD on the version ring (Sec. 3.1 updates under the
-// SSP / ESSP read schedule): the fused per-clock kernel, the kernel for the
-// entries of very active users, and the objective.
-#include <cfloat>
+// SSP / ESSP read schedule).  One clock is:
+//   sgd_chunks_kernel   entries of very active users, in chunks (if any);
+//   sgd_users_kernel    every other user: its row of version c, written once;
+//   heavy_merge_kernel  rows of the very active users (if any);
+//   item_merge_kernel   the Clock() merge of the item rows.
+// Item-row (and heavy-user) deltas are summed, unscaled, into zero-initialised
+// replica rows so that popular rows spread their fp32 reductions over many
+// L2 addresses; the merges apply eta, the hot-row scale and the sum of the
+// replicas, then clear them for the next clock.
+#include <algorithm>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -31,77 +38,149 @@ __device__ __forceinline__ float4 f4_zero() { return make_float4(0.f, 0.f, 0.f, 
 
 __device__ __forceinline__ float dot4(float4 a, float4 b) { return a.x * b.x + a.y * b.y + a.z * b.z + a.w * b.w; }
 
-// Entries processed per batch of independent R-row gathers.
-constexpr int kBatch = 4;
+__device__ __forceinline__ float4 f4_axpy(float s, float4 x, float4 y) {  // y + s x
+  return make_float4(y.x + s * x.x, y.y + s * x.y, y.z + s * x.z, y.w + s * x.w);
+}
 
-// Process entries [beg, end) of one user whose read-version row is Lv (lane
-// slices of NV float4).  Accumulates the user's summed gradient term
-// sum(e R_j - lambda L_i) into gL and issues every item row's scaled update
-// eta s_j (e L_i - lambda R_j) into version c.  Returns the sum of e^2 on the
-// group's lane 0.
-template <int G, int NV>
-__device__ __forceinline__ float process_entries(const SgdArgs& a, int32_t beg, int32_t end, const float4 (&Lv)[NV],
-                                                 float4 (&gL)[NV], const float4* __restrict__ Rv_base,
-                                                 float4* __restrict__ Rout_base, int glane, unsigned gmask,
-                                                 int32_t K4) {
-  float loss = 0.f;
-  for (int32_t t0 = beg; t0 < end; t0 += G) {
-    // Lane l of the group fetches entry t0 + l and its item's scale.
-    const int32_t nb = min(G, end - t0);
-    int32_t my_j = 0;
-    float my_d = 0.f, my_s = 1.f;
-    if (glane < nb) {
-      my_j = a.rec_j[t0 + glane];
-      my_d = a.rec_D[t0 + glane];
-      if (a.cap > 0) {
-        const int32_t cnt = a.item_cnt[my_j];
-        if (cnt > a.cap) my_s = (float)a.cap / (float)cnt;
-      }
+// Scale of a row's summed update under the hot-row step cap.
+__device__ __forceinline__ float cap_scale(int32_t cap, int32_t n) {
+  return (cap > 0 && n > cap) ? (float)cap / (float)n : 1.f;
+}
+
+// Entry t of the minibatch (item, value); zeros past the end.
+__device__ __forceinline__ void load_entry(const SgdArgs& a, int32_t t, int32_t& j, float& d) {
+  if (t < a.n_b) {
+    j = __ldg(a.rec_j + t);
+    d = __ldg(a.rec_D + t);
+  } else {
+    j = 0;
+    d = 0.f;
+  }
+}
+
+// Replica row of item j that entry t adds into.
+__device__ __forceinline__ int32_t replica_row(const SgdArgs& a, int32_t t, int32_t j) {
+  const int32_t r0 = __ldg(a.item_rep + j), r1 = __ldg(a.item_rep + j + 1);
+  return r0 + (t & (r1 - r0 - 1));
+}
+
+// A group's sliding window over the minibatch entries: lane l holds entry
+// W + l (cur) and W + G + l (nxt, prefetched).
+template <int G>
+struct Window {
+  int32_t W;
+  int32_t cj, cdst, nj;
+  float cd, nd;
+
+  __device__ __forceinline__ void reload(const SgdArgs& a, int32_t start, int glane) {
+    W = start;
+    load_entry(a, W + glane, cj, cd);
+    cdst = replica_row(a, W + glane, cj);
+    load_entry(a, W + G + glane, nj, nd);
+  }
+  // Make entry t (>= W) part of cur.
+  __device__ __forceinline__ void cover(const SgdArgs& a, int32_t t, int glane) {
+    if (t < W + G) return;
+    if (t < W + 2 * G) {
+      W += G;
+      cj = nj;
+      cd = nd;
+      cdst = replica_row(a, W + glane, cj);
+      load_entry(a, W + G + glane, nj, nd);
+    } else {
+      reload(a, t, glane);
     }
-    for (int32_t b0 = 0; b0 < nb; b0 += kBatch) {
-      int32_t jj[kBatch];
-      float4 R[kBatch][NV];
+  }
+};
+
+// Entries [t0, t0 + nbat) of one row group, all inside the window's cur part
+// and all of one user whose read-version row is Lv.  For each entry:
+// e = D - L.R at the read version; gL += e R - lambda L; the item update
+// e L - lambda R goes (unscaled) into the entry's replica row of dR.
+template <int G, int NV, int B>
+__device__ __forceinline__ void process_batch(const SgdArgs& a, const Window<G>& win, int32_t t0, int32_t nbat,
+                                              const float4 (&Lv)[NV], float4 (&gL)[NV],
+                                              const float4* __restrict__ Rv_base, float4* __restrict__ dR4,
+                                              int glane, unsigned gmask, int32_t K4, float& loss) {
+  const int32_t i0 = t0 - win.W;
+  int32_t jj[B];
+  float4 R[B][NV];
 #pragma unroll
-      for (int u = 0; u < kBatch; ++u) {
-        jj[u] = __shfl_sync(gmask, my_j, b0 + u, G);
+  for (int u = 0; u < B; ++u) {
+    jj[u] = __shfl_sync(gmask, win.cj, (i0 + u) & (G - 1), G);
 #pragma unroll
-        for (int t = 0; t < NV; ++t) {
-          const int32_t q = glane + t * G;
-          R[u][t] = (b0 + u < nb && q < K4) ? Rv_base[(int64_t)jj[u] * K4 + q] : f4_zero();
-        }
-      }
+    for (int t = 0; t < NV; ++t) {
+      const int32_t q = glane + t * G;
+      R[u][t] = (u < nbat && q < K4) ? __ldg(Rv_base + (int64_t)jj[u] * K4 + q) : f4_zero();
+    }
+  }
 #pragma unroll
-      for (int u = 0; u < kBatch; ++u) {
-        const float d = __shfl_sync(gmask, my_d, b0 + u, G);
-        const float sj = __shfl_sync(gmask, my_s, b0 + u, G);
-        if (b0 + u >= nb) break;
-        float part = 0.f;
+  for (int u = 0; u < B; ++u) {
+    const float d = __shfl_sync(gmask, win.cd, (i0 + u) & (G - 1), G);
+    const int32_t dst = __shfl_sync(gmask, win.cdst, (i0 + u) & (G - 1), G);
+    if (u < nbat) {
+      float part = 0.f;
 #pragma unroll
-        for (int t = 0; t < NV; ++t) part += dot4(Lv[t], R[u][t]);
-        const float e = d - group_sum<G>(part, gmask);
-        loss += e * e;
-        const float ce = a.eta * sj * e, cl = a.eta * sj * a.lambda;
+      for (int t = 0; t < NV; ++t) part += dot4(Lv[t], R[u][t]);
+      const float e = d - group_sum<G>(part, gmask);
+      loss += e * e;
 #pragma unroll
-        for (int t = 0; t < NV; ++t) {
-          const int32_t q = glane + t * G;
-          if (q < K4) {
-            const float4 r = R[u][t], l = Lv[t];
-            gL[t].x += e * r.x - a.lambda * l.x;
-            gL[t].y += e * r.y - a.lambda * l.y;
-            gL[t].z += e * r.z - a.lambda * l.z;
-            gL[t].w += e * r.w - a.lambda * l.w;
-            red_add_v4(Rout_base + (int64_t)jj[u] * K4 + q,
-                       make_float4(ce * l.x - cl * r.x, ce * l.y - cl * r.y, ce * l.z - cl * r.z,
-                                   ce * l.w - cl * r.w));
-          }
+      for (int t = 0; t < NV; ++t) {
+        const int32_t q = glane + t * G;
+        if (q < K4) {
+          const float4 r = R[u][t], l = Lv[t];
+          gL[t].x += e * r.x - a.lambda * l.x;
+          gL[t].y += e * r.y - a.lambda * l.y;
+          gL[t].z += e * r.z - a.lambda * l.z;
+          gL[t].w += e * r.w - a.lambda * l.w;
+          red_add_v4(dR4 + (int64_t)dst * K4 + q, make_float4(e * l.x - a.lambda * r.x, e * l.y - a.lambda * r.y,
+                                                              e * l.z - a.lambda * r.z, e * l.w - a.lambda * r.w));
         }
       }
     }
   }
-  return loss;
 }
 
-template <int G>
+// All entries [beg, end) of one user (or chunk), batch by batch.
+template <int G, int NV, int B>
+__device__ __forceinline__ void process_range(const SgdArgs& a, Window<G>& win, int32_t beg, int32_t end,
+                                              const float4 (&Lv)[NV], float4 (&gL)[NV],
+                                              const float4* __restrict__ Rv_base, float4* __restrict__ dR4,
+                                              int glane, unsigned gmask, int32_t K4, float& loss) {
+  for (int32_t t0 = beg; t0 < end;) {
+    win.cover(a, t0, glane);
+    const int32_t nbat = min(B, min(end - t0, win.W + G - t0));
+    process_batch<G, NV, B>(a, win, t0, nbat, Lv, gL, Rv_base, dR4, glane, gmask, K4, loss);
+    t0 += nbat;
+  }
+}
+
+__device__ __forceinline__ float4 f4_add(float4 a, float4 b) {
+  return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+
+// Sum of n replica slices p[0], p[stride], ..., each cleared after reading;
+// eight independent loads in flight per lane.
+__device__ __forceinline__ float4 sum_and_clear(float4* p, int32_t n, int32_t stride) {
+  float4 acc = f4_zero();
+  int32_t r = 0;
+  for (; r + 8 <= n; r += 8) {
+    float4 x[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) x[k] = p[(int64_t)(r + k) * stride];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      p[(int64_t)(r + k) * stride] = f4_zero();
+      acc = f4_add(acc, x[k]);
+    }
+  }
+  for (; r < n; ++r) {
+    acc = f4_add(acc, p[(int64_t)r * stride]);
+    p[(int64_t)r * stride] = f4_zero();
+  }
+  return acc;
+}
+
 __device__ __forceinline__ void flush_loss(double* out, float v, int lane) {
   if (out == nullptr) return;
   double x = (double)v;
@@ -112,70 +191,109 @@ __device__ __forceinline__ void flush_loss(double* out, float v, int lane) {
 
 }  // namespace
 
-// One row group per user: L_i^c = L_i^{base} + eta s_i sum_k (e_k R_j - lambda L_i),
-// written once (no atomics); every entry's item update goes to version c by
-// a vector reduction at L2.  Users with more than kHeavy entries only get the
-// copy here; their entries are handled by sgd_chunks_kernel afterwards.
-template <int G, int NV>
+// Each warp takes 32 consecutive users (one coalesced metadata load); a row
+// group of G lanes walks G of them in order, prefetching the next user's rows
+// and the next window of entries while it computes the current user.
+//   L_i^c = L_i^base + eta s_i sum_k (e_k R_j - lambda L_i)   (written once)
+// Users with more than kHeavy entries are left to the chunk / heavy-merge path.
+template <int G, int NV, int B>
 __global__ void __launch_bounds__(256) sgd_users_kernel(SgdArgs a) {
   const int lane = threadIdx.x & 31;
   const int glane = lane & (G - 1);
+  const int grp = lane / G;
   const unsigned gmask = group_mask<G>(lane);
   const int32_t K4 = a.K >> 2;
   const int64_t slot4 = a.n_rows * K4;
   float4* ring4 = reinterpret_cast<float4*>(a.ring);
   float4* out4 = ring4 + (int64_t)a.slot_out * slot4;
+  const float4* base4 = ring4 + (int64_t)a.slot_base * slot4;
+  float4* dR4 = reinterpret_cast<float4*>(a.dR);
   const uint64_t pol = policy_evict_first();
   float loss = 0.f;
-  // Groups of a warp stay together across the loop (uniform trip count).
-  const int64_t warp_first = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * (32 / G);
+  const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t ubase = warp_first; ubase < a.n_users; ubase += nwarps * (32 / G)) {
-    const int64_t u = ubase + lane / G;
-    if (u < a.n_users) {
-      const int32_t vs = a.v[a.worker[u]] % a.nslots;
-      const int32_t beg = a.uoff[u], end = a.uoff[u + 1];
-      const float4* Lv_row = ring4 + (int64_t)vs * slot4 + u * K4;
-      const float4* Lb_row = ring4 + (int64_t)a.slot_base * slot4 + u * K4;
-      float4 Lv[NV], Lb[NV], gL[NV];
+
+  for (int64_t u0 = warp_id * 32; u0 < a.n_users; u0 += nwarps * 32) {
+    const int64_t uu = u0 + lane;
+    int32_t m_beg = 0, m_end = 0, m_vs = 0;
+    if (uu < a.n_users) {
+      m_beg = __ldg(a.uoff + uu);
+      m_end = __ldg(a.uoff + uu + 1);
+      m_vs = __ldg(a.v + __ldg(a.worker + uu)) % a.nslots;
+    }
+    const int64_t g0 = u0 + (int64_t)grp * G;
+    const int32_t nusers = (int32_t)max((int64_t)0, min((int64_t)G, (int64_t)a.n_users - g0));
+    if (nusers == 0) continue;
+
+    Window<G> win;
+    win.reload(a, __shfl_sync(gmask, m_beg, 0, G), glane);
+
+    // rows of the group's first user
+    int32_t nvs = __shfl_sync(gmask, m_vs, 0, G);
+    int32_t nbeg = __shfl_sync(gmask, m_beg, 0, G);
+    int32_t nend = __shfl_sync(gmask, m_end, 0, G);
+    float4 Lvn[NV], Lbn[NV];
+    bool nsame;
+    {
+      const int32_t n = nend - nbeg;
+      nsame = (nvs == a.slot_base) && n > 0;
 #pragma unroll
       for (int t = 0; t < NV; ++t) {
         const int32_t q = glane + t * G;
-        Lv[t] = q < K4 ? ld_stream(Lv_row + q, pol) : f4_zero();
-        gL[t] = f4_zero();
+        const bool in = q < K4 && n <= kHeavy;
+        Lvn[t] = (in && n > 0) ? ld_stream(ring4 + (int64_t)nvs * slot4 + g0 * K4 + q, pol) : f4_zero();
+        Lbn[t] = (in && !nsame) ? ld_stream(base4 + g0 * K4 + q, pol) : f4_zero();
       }
+    }
+
+    for (int32_t t = 0; t < nusers; ++t) {
+      const int64_t u = g0 + t;
+      const int32_t vs = nvs, beg = nbeg, end = nend;
+      const bool same = nsame;
+      float4 Lv[NV], Lb[NV];
 #pragma unroll
-      for (int t = 0; t < NV; ++t) {
-        const int32_t q = glane + t * G;
-        Lb[t] = (vs == a.slot_base || q >= K4) ? Lv[t] : ld_stream(Lb_row + q, pol);
+      for (int k = 0; k < NV; ++k) {
+        Lv[k] = Lvn[k];
+        Lb[k] = Lbn[k];
+      }
+      if (t + 1 < nusers) {  // prefetch the next user's rows
+        nvs = __shfl_sync(gmask, m_vs, t + 1, G);
+        nbeg = __shfl_sync(gmask, m_beg, t + 1, G);
+        nend = __shfl_sync(gmask, m_end, t + 1, G);
+        const int32_t n = nend - nbeg;
+        nsame = (nvs == a.slot_base) && n > 0;
+#pragma unroll
+        for (int k = 0; k < NV; ++k) {
+          const int32_t q = glane + k * G;
+          const bool in = q < K4 && n <= kHeavy;
+          Lvn[k] = (in && n > 0) ? ld_stream(ring4 + (int64_t)nvs * slot4 + (u + 1) * K4 + q, pol) : f4_zero();
+          Lbn[k] = (in && !nsame) ? ld_stream(base4 + (u + 1) * K4 + q, pol) : f4_zero();
+        }
       }
       const int32_t n = end - beg;
-      float scale = 0.f;
-      if (n <= kHeavy) {
-        const float4* Rv_base = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4;
-        float4* Rout_base = out4 + (int64_t)a.n_users * K4;
-        loss += process_entries<G, NV>(a, beg, end, Lv, gL, Rv_base, Rout_base, glane, gmask, K4);
-        scale = a.eta * ((a.cap > 0 && n > a.cap) ? (float)a.cap / (float)n : 1.f);
-      }
-      float4* Lo_row = out4 + u * K4;
+      if (n > kHeavy) continue;
+      float4 gL[NV];
 #pragma unroll
-      for (int t = 0; t < NV; ++t) {
-        const int32_t q = glane + t * G;
-        if (q < K4) {
-          const float4 b = Lb[t], g = gL[t];
-          st_stream(Lo_row + q, make_float4(b.x + scale * g.x, b.y + scale * g.y, b.z + scale * g.z, b.w + scale * g.w),
-                    pol);
-        }
+      for (int k = 0; k < NV; ++k) gL[k] = f4_zero();
+      if (n > 0) {
+        const float4* Rv_base = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4;
+        process_range<G, NV, B>(a, win, beg, end, Lv, gL, Rv_base, dR4, glane, gmask, K4, loss);
+      }
+      const float sc = a.eta * cap_scale(a.cap, n);
+#pragma unroll
+      for (int k = 0; k < NV; ++k) {
+        const int32_t q = glane + k * G;
+        if (q < K4) st_stream(out4 + u * K4 + q, f4_axpy(sc, gL[k], same ? Lv[k] : Lb[k]), pol);
       }
     }
   }
-  flush_loss<G>(a.sq_loss, glane == 0 ? loss : 0.f, lane);
+  flush_loss(a.sq_loss, glane == 0 ? loss : 0.f, lane);
 }
 
-// Entries of users with more than kHeavy entries in the minibatch, split in
-// chunks of at most kChunk entries; each chunk adds its partial user update
-// to version c by vector reductions (after sgd_users_kernel copied the row).
-template <int G, int NV>
+// Chunks of at most kChunk entries of users with more than kHeavy entries:
+// the chunk's partial user update sum (e R - lambda L) goes, unscaled, into
+// one of its user's replica rows of dL; item updates as in the user kernel.
+template <int G, int NV, int B>
 __global__ void __launch_bounds__(256) sgd_chunks_kernel(ChunkArgs c) {
   const SgdArgs& a = c.a;
   const int lane = threadIdx.x & 31;
@@ -183,42 +301,85 @@ __global__ void __launch_bounds__(256) sgd_chunks_kernel(ChunkArgs c) {
   const unsigned gmask = group_mask<G>(lane);
   const int32_t K4 = a.K >> 2;
   const int64_t slot4 = a.n_rows * K4;
-  float4* ring4 = reinterpret_cast<float4*>(a.ring);
-  float4* out4 = ring4 + (int64_t)a.slot_out * slot4;
+  const float4* ring4 = reinterpret_cast<const float4*>(a.ring);
+  float4* dR4 = reinterpret_cast<float4*>(a.dR);
+  float4* dL4 = reinterpret_cast<float4*>(c.dL);
   float loss = 0.f;
-  const int64_t warp_first = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * (32 / G);
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t kbase = warp_first; kbase < c.n_chunks; kbase += nwarps * (32 / G)) {
-    const int64_t k = kbase + lane / G;
+  const int64_t first = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * (32 / G);
+  const int64_t step = (((int64_t)gridDim.x * blockDim.x) >> 5) * (32 / G);
+  for (int64_t kb = first; kb < c.n_chunks; kb += step) {
+    const int64_t k = kb + lane / G;
     if (k < c.n_chunks) {
-      const int32_t u = c.chunk_user[k];
-      const int32_t vs = a.v[a.worker[u]] % a.nslots;
-      const float4* Lv_row = ring4 + (int64_t)vs * slot4 + (int64_t)u * K4;
+      const int4 ch = c.chunk[k];
+      const int32_t vs = __ldg(a.v + __ldg(a.worker + ch.x)) % a.nslots;
+      const float4* Lrow = ring4 + (int64_t)vs * slot4 + (int64_t)ch.x * K4;
       float4 Lv[NV], gL[NV];
 #pragma unroll
       for (int t = 0; t < NV; ++t) {
         const int32_t q = glane + t * G;
-        Lv[t] = q < K4 ? Lv_row[q] : f4_zero();
+        Lv[t] = q < K4 ? Lrow[q] : f4_zero();
         gL[t] = f4_zero();
       }
+      Window<G> win;
+      win.reload(a, ch.y, glane);
       const float4* Rv_base = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4;
-      float4* Rout_base = out4 + (int64_t)a.n_users * K4;
-      loss += process_entries<G, NV>(a, c.chunk_begin[k], c.chunk_end[k], Lv, gL, Rv_base, Rout_base, glane, gmask,
-                                     K4);
-      const int32_t n = a.uoff[u + 1] - a.uoff[u];
-      const float scale = a.eta * ((a.cap > 0 && n > a.cap) ? (float)a.cap / (float)n : 1.f);
-      float4* Lo_row = out4 + (int64_t)u * K4;
+      process_range<G, NV, B>(a, win, ch.y, ch.z, Lv, gL, Rv_base, dR4, glane, gmask, K4, loss);
 #pragma unroll
       for (int t = 0; t < NV; ++t) {
         const int32_t q = glane + t * G;
-        if (q < K4) {
-          const float4 g = gL[t];
-          red_add_v4(Lo_row + q, make_float4(scale * g.x, scale * g.y, scale * g.z, scale * g.w));
-        }
+        if (q < K4) red_add_v4(dL4 + (int64_t)ch.w * K4 + q, gL[t]);
       }
     }
   }
-  flush_loss<G>(a.sq_loss, glane == 0 ? loss : 0.f, lane);
+  flush_loss(a.sq_loss, glane == 0 ? loss : 0.f, lane);
+}
+
+// Heavy user rows: L^c = L^base + eta s sum of the user's replica rows (row u
+// of dL, then rows hv.y .. hv.y + hv.z - 2); the replicas are cleared for the
+// next clock.  One warp per heavy user.
+__global__ void __launch_bounds__(256) heavy_merge_kernel(HeavyMergeArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int32_t K4 = a.K >> 2;
+  const int64_t slot4 = a.n_rows * K4;
+  float4* ring4 = reinterpret_cast<float4*>(a.ring);
+  float4* dL4 = reinterpret_cast<float4*>(a.dL);
+  for (int64_t h = warp; h < a.n_heavy; h += nwarps) {
+    const int4 hv = a.heavy[h];
+    const float sc = a.eta * cap_scale(a.cap, hv.w);
+    for (int32_t q = lane; q < K4; q += 32) {
+      float4* p0 = dL4 + (int64_t)hv.x * K4 + q;
+      float4 acc = *p0;
+      *p0 = f4_zero();
+      acc = f4_add(acc, sum_and_clear(dL4 + (int64_t)hv.y * K4 + q, hv.z - 1, K4));
+      const float4 b = ring4[(int64_t)a.slot_base * slot4 + (int64_t)hv.x * K4 + q];
+      ring4[(int64_t)a.slot_out * slot4 + (int64_t)hv.x * K4 + q] = f4_axpy(sc, acc, b);
+    }
+  }
+}
+
+// Clock() merge of the item rows (Sec. 2.1 additive updates, Sec. 4 server
+// clock): R^c_j = R^base_j + eta s_j sum of j's replica rows; replicas
+// cleared.  One warp per item.
+__global__ void __launch_bounds__(256) item_merge_kernel(ItemMergeArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int32_t K4 = a.K >> 2;
+  const int64_t slot4 = a.n_rows * K4;
+  float4* ring4 = reinterpret_cast<float4*>(a.ring);
+  float4* dR4 = reinterpret_cast<float4*>(a.dR);
+  for (int64_t j = warp; j < a.n_items; j += nwarps) {
+    const int32_t r0 = __ldg(a.item_rep + j), r1 = __ldg(a.item_rep + j + 1);
+    const float sc = a.eta * cap_scale(a.cap, __ldg(a.item_cnt + j));
+    const int64_t row = (int64_t)a.n_users + j;
+    for (int32_t q = lane; q < K4; q += 32) {
+      const float4 acc = sum_and_clear(dR4 + (int64_t)r0 * K4 + q, r1 - r0, K4);
+      const float4 b = ring4[(int64_t)a.slot_base * slot4 + row * K4 + q];
+      ring4[(int64_t)a.slot_out * slot4 + row * K4 + q] = f4_axpy(sc, acc, b);
+    }
+  }
 }
 
 namespace {
@@ -234,29 +395,32 @@ int sm_count() {
   return sms;
 }
 
-template <int G, int NV>
-cudaError_t launch_users_t(const SgdArgs& a, cudaStream_t st) {
-  const int threads = 256;
-  const int64_t groups_per_block = threads / G;
-  const int64_t want = (a.n_users + groups_per_block - 1) / groups_per_block;
-  const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sm_count() * 8));
-  sgd_users_kernel<G, NV><<<blocks, threads, 0, st>>>(a);
-  return cudaGetLastError();
+int grid_for(int64_t work_items, int64_t per_block, int max_per_sm) {
+  const int64_t want = (work_items + per_block - 1) / per_block;
+  return (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sm_count() * max_per_sm));
 }
 
-template <int G, int NV>
-cudaError_t launch_chunks_t(const ChunkArgs& c, cudaStream_t st) {
-  if (c.n_chunks <= 0) return cudaSuccess;
-  const int threads = 256;
-  const int64_t groups_per_block = threads / G;
-  const int64_t want = (c.n_chunks + groups_per_block - 1) / groups_per_block;
-  const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sm_count() * 8));
-  sgd_chunks_kernel<G, NV><<<blocks, threads, 0, st>>>(c);
-  return cudaGetLastError();
-}
+constexpr int kBatchEntries = 4;
 
-// Row-group shape for K values: G lanes per row (power of two <= 32), NV
-// float4 per lane.  K is a multiple of 4 in [4, 512].
+template <int G, int NV>
+struct UsersF {
+  static cudaError_t run(const SgdArgs& a, cudaStream_t st) {
+    // 8 warps per block, 32 users per warp
+    sgd_users_kernel<G, NV, kBatchEntries><<<grid_for(a.n_users, 256, 8), 256, 0, st>>>(a);
+    return cudaGetLastError();
+  }
+};
+template <int G, int NV>
+struct ChunksF {
+  static cudaError_t run(const ChunkArgs& c, cudaStream_t st) {
+    if (c.n_chunks <= 0) return cudaSuccess;
+    sgd_chunks_kernel<G, NV, kBatchEntries><<<grid_for(c.n_chunks, 256 / G, 8), 256, 0, st>>>(c);
+    return cudaGetLastError();
+  }
+};
+
+// Row-group shape for K: G lanes per row (power of two <= 32), NV float4 per
+// lane.  K is a multiple of 4 in [4, 512].
 template <template <int, int> class F, typename Arg>
 cudaError_t dispatch_k(int32_t K, const Arg& a, cudaStream_t st) {
   const int32_t K4 = K / 4;
@@ -271,19 +435,22 @@ cudaError_t dispatch_k(int32_t K, const Arg& a, cudaStream_t st) {
   return F<32, 4>::run(a, st);
 }
 
-template <int G, int NV>
-struct UsersF {
-  static cudaError_t run(const SgdArgs& a, cudaStream_t st) { return launch_users_t<G, NV>(a, st); }
-};
-template <int G, int NV>
-struct ChunksF {
-  static cudaError_t run(const ChunkArgs& a, cudaStream_t st) { return launch_chunks_t<G, NV>(a, st); }
-};
-
 }  // namespace
 
 cudaError_t launch_sgd_users(const SgdArgs& a, cudaStream_t st) { return dispatch_k<UsersF>(a.K, a, st); }
 cudaError_t launch_sgd_chunks(const ChunkArgs& c, cudaStream_t st) { return dispatch_k<ChunksF>(c.a.K, c, st); }
+
+cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st) {
+  if (a.n_heavy <= 0) return cudaSuccess;
+  heavy_merge_kernel<<<grid_for(a.n_heavy, 8, 8), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_item_merge(const ItemMergeArgs& a, cudaStream_t st) {
+  if (a.n_items <= 0) return cudaSuccess;
+  item_merge_kernel<<<grid_for(a.n_items, 8, 16), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
 
 // ---------------------------------------------------------------------------
 // Objective (Sec. 3.1, Sec. 5) over all entries: sum e^2 and
@@ -328,13 +495,13 @@ __global__ void __launch_bounds__(256) objective_kernel(const float* __restrict_
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    double a = 0.0, b = 0.0;
+    double x = 0.0, y = 0.0;
     for (int i = 0; i < (int)(blockDim.x >> 5); ++i) {
-      a += sh[0][i];
-      b += sh[1][i];
+      x += sh[0][i];
+      y += sh[1][i];
     }
-    atomicAdd(out2, a);
-    atomicAdd(out2 + 1, b);
+    atomicAdd(out2, x);
+    atomicAdd(out2 + 1, y);
   }
 }
 
@@ -342,10 +509,7 @@ cudaError_t launch_objective(const float* slot, int64_t n_users, int32_t K, cons
                              const float* rec_D, int64_t n_obs, float lambda, double* out2, cudaStream_t st) {
   cudaError_t err = cudaMemsetAsync(out2, 0, 2 * sizeof(double), st);
   if (err != cudaSuccess || n_obs == 0) return err;
-  const int threads = 256;
-  const int64_t want = (n_obs + 7) / 8;
-  const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sm_count() * 16));
-  objective_kernel<<<blocks, threads, 0, st>>>(slot, n_users, K, rec_u, rec_j, rec_D, n_obs, lambda, out2);
+  objective_kernel<<<grid_for(n_obs, 8, 16), 256, 0, st>>>(slot, n_users, K, rec_u, rec_j, rec_D, n_obs, lambda, out2);
   return cudaGetLastError();
 }
 
