@@ -220,6 +220,24 @@ esspt_status esspt_mf_stage_minibatch(esspt_ctx* ctx, int32_t b, const int32_t* 
  * after `after`.  NULL, NULL turns it off. */
 esspt_status esspt_set_profile_events(esspt_ctx* ctx, void* before, void* after);
 
+/* The objective of esspt_mf_objective() split by worker, for callers that
+ * cannot allocate device memory (a pool owned by another framework, a hook
+ * inside a hot loop, a fixed memory budget).  It needs neither the caller's
+ * scratch nor any allocation: its accumulators are a 32 KB array built into
+ * the library, held by every GPU that loads it until the process exits.
+ * The paper has no counterpart to this entry point.
+ *   version  a final version in the live window (as esspt_mf_objective);
+ *   h_sq, h_pen  host, P doubles each: per worker p, sum e^2 and
+ *            sum [e^2 + lambda(|L_i|^2 + |R_j|^2)] over the entries of the
+ *            users p owns.
+ * At most 2048 workers; more gives ESSPT_EINVAL and queues no work.  The first
+ * call on a device looks up the array's address with that device current;
+ * make it before any stream capture.  Every call clears the shared array
+ * first and synchronises the stream; calls that overlap on the GPU (other
+ * streams, no ordering between them) race on the array. */
+esspt_status esspt_mf_worker_objective_noalloc(esspt_ctx* ctx, int32_t version, float lambda, double* h_sq,
+                                               double* h_pen);
+
 #ifdef __cplusplus
 }
 #endif

@@ -203,6 +203,33 @@ bool mf_sizes_ok(const esspt_ctx* c, int64_t n_obs, int64_t n_users, int32_t F) 
 
 }  // namespace
 
+namespace esspt {
+
+esspt_status mf_view(esspt_ctx* c, int32_t version, const float** slot, int64_t* n_users, int32_t* K,
+                     const int32_t** rec_u, const int32_t** rec_j, const float** rec_D, const int32_t** worker,
+                     int64_t* n_obs, int32_t* P, cudaStream_t* st) {
+  esspt_status s = need_init(c);
+  if (s != ESSPT_OK) return s;
+  if (!c->mf) return fail(c, ESSPT_ESTATE, "no MF data loaded (call esspt_mf_load)");
+  const int32_t lo = c->clock - 1 - c->s > 0 ? c->clock - 1 - c->s : 0;
+  if (version < lo || version > c->clock - 1) return fail(c, ESSPT_EINVAL, "version outside the live window");
+  *slot = slot_ptr(c, version);
+  *n_users = c->n_users;
+  *K = c->K;
+  *rec_u = c->rec_u;
+  *rec_j = c->rec_j;
+  *rec_D = c->rec_D;
+  *worker = c->worker;
+  *n_obs = c->n_obs;
+  *P = c->P;
+  *st = c->st;
+  return ESSPT_OK;
+}
+
+esspt_status mf_fail(esspt_ctx* c, esspt_status code, const char* msg) { return fail(c, code, msg); }
+
+}  // namespace esspt
+
 extern "C" {
 
 size_t esspt_workspace_bytes(const esspt_config* cfg) {

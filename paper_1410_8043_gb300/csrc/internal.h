@@ -145,4 +145,12 @@ int64_t layout_max_user_reps(int64_t n_obs);
 cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st);
 cudaError_t launch_validate(const LayoutBuild& b, cudaStream_t st);
 
+// Read-only view of a context's loaded MF entries and of table version
+// `version` (checked against the live window), for entry points defined in
+// other translation units; and the context's error setter.
+esspt_status mf_view(esspt_ctx* ctx, int32_t version, const float** slot, int64_t* n_users, int32_t* K,
+                     const int32_t** rec_u, const int32_t** rec_j, const float** rec_D, const int32_t** worker,
+                     int64_t* n_obs, int32_t* P, cudaStream_t* st);
+esspt_status mf_fail(esspt_ctx* ctx, esspt_status code, const char* msg);
+
 }  // namespace esspt

@@ -26,7 +26,7 @@ EXPORTS = (
     "esspt_clock", "esspt_set_schedule", "esspt_poll", "esspt_read_schedule", "esspt_read_table",
     "esspt_last_error", "esspt_mf_workspace_bytes", "esspt_mf_scratch_bytes", "esspt_mf_load",
     "esspt_mf_sgd_clock", "esspt_mf_objective", "esspt_mf_minibatch_size", "esspt_mf_export_minibatch",
-    "esspt_mf_stage_minibatch", "esspt_set_profile_events",
+    "esspt_mf_stage_minibatch", "esspt_set_profile_events", "esspt_mf_worker_objective_noalloc",
 )
 
 
@@ -85,6 +85,7 @@ def lib() -> ctypes.CDLL:
         "esspt_mf_export_minibatch": (ctypes.c_int, [P, I32, P, P, P, P]),
         "esspt_mf_stage_minibatch": (ctypes.c_int, [P, I32, P, P, P, P]),
         "esspt_set_profile_events": (ctypes.c_int, [P, P, P]),
+        "esspt_mf_worker_objective_noalloc": (ctypes.c_int, [P, I32, ctypes.c_float, P, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -279,6 +280,14 @@ class Table:
             self._check(lib().esspt_set_profile_events(self._h, None, None))
         else:
             self._check(lib().esspt_set_profile_events(self._h, before.cuda_event, after.cuda_event))
+
+    def mf_worker_objective_noalloc(self, version: int, lam: float):
+        """esspt_mf_worker_objective_noalloc: per-worker (sum e^2, penalised sum)
+        as two float64[P] arrays, computed without any device allocation."""
+        sq = np.empty(self.P, dtype=np.float64)
+        pen = np.empty(self.P, dtype=np.float64)
+        self._check(lib().esspt_mf_worker_objective_noalloc(self._h, version, lam, sq.ctypes.data, pen.ctypes.data))
+        return sq, pen
 
     @classmethod
     def for_workload(cls, w, data, partition, **kw) -> "Table":
