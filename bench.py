@@ -116,26 +116,30 @@ def _barrier(world):
         dist.barrier()
 
 
-def _max_over_ranks(world, x: float) -> float:
+def _reduce_over_ranks(world, x: float, op: str) -> float:
+    """Max or sum of a host scalar over the ranks (NCCL on GPUs, gloo on CPU)."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
 
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX if op == "max" else dist.ReduceOp.SUM)
     return float(t.item())
+
+
+def _max_over_ranks(world, x: float) -> float:
+    return _reduce_over_ranks(world, x, "max")
 
 
 def _sum_over_ranks(world, x: float) -> float:
-    if world == 1:
-        return x
-    import torch
-    import torch.distributed as dist
+    return _reduce_over_ranks(world, x, "sum")
 
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t)
-    return float(t.item())
+
+def replica_throughput(world, ratings: float, ms: float) -> float:
+    """Whole-job ratings/s of N independent replicas: all ratings over the slowest rank's time."""
+    return _sum_over_ranks(world, ratings) / (_max_over_ranks(world, ms) / 1e3)
 
 
 class FloorModel:
@@ -242,7 +246,7 @@ def run_gpu(args, w):
     ms_max = _max_over_ranks(world, ms)
     ratings = float(sum(counts))
     total_ratings = _sum_over_ranks(world, ratings)
-    value = total_ratings / (ms_max / 1e3)
+    value = replica_throughput(world, ratings, ms)
     c_final = t.clock_index - 1
     sq, pen = t.mf_objective(c_final, w.lam)
 

@@ -28,7 +28,7 @@ struct esspt_ctx {
   int64_t n_users = 0, n_items = 0, n_obs = 0;
   int32_t F = 0;
   int32_t *rec_u = nullptr, *rec_j = nullptr, *uoff = nullptr, *item_cnt = nullptr, *worker = nullptr;
-  int32_t* item_rep = nullptr;
+  int32_t *item_rep = nullptr, *rec_dst = nullptr;
   float *rec_D = nullptr, *dR = nullptr, *dL = nullptr;
   int4 *chunk = nullptr, *heavy = nullptr;
   std::vector<int64_t> mb_base, chunk_base, heavy_base;
@@ -157,7 +157,7 @@ bool is_host_ptr(const void* p) {
 }
 
 struct MfCarve {
-  size_t rec_u, rec_j, rec_D, uoff, mb_base, item_cnt, item_rep, dR, worker, chunk, chunk_base, heavy, heavy_base, dL,
+  size_t rec_u, rec_j, rec_D, rec_dst, uoff, mb_base, item_cnt, item_rep, dR, worker, chunk, chunk_base, heavy, heavy_base, dL,
       total;
   int64_t max_chunks, max_heavy, dR_rows, dL_rows;
 };
@@ -181,6 +181,7 @@ MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int
   k.rec_u = take(sizeof(int32_t) * (n_obs + 4));
   k.rec_j = take(sizeof(int32_t) * (n_obs + 4));
   k.rec_D = take(sizeof(float) * (n_obs + 4));
+  k.rec_dst = take(sizeof(int32_t) * (n_obs + 4));
   k.uoff = take(sizeof(int32_t) * (size_t)F * (n_users + 1));
   k.mb_base = take(sizeof(int64_t) * (F + 1));
   k.item_cnt = take(sizeof(int32_t) * (size_t)F * n_items);
@@ -433,6 +434,7 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   b.mb_base = reinterpret_cast<int64_t*>(w + k.mb_base);
   b.item_cnt = reinterpret_cast<int32_t*>(w + k.item_cnt);
   b.item_rep = reinterpret_cast<int32_t*>(w + k.item_rep);
+  b.rec_dst = reinterpret_cast<int32_t*>(w + k.rec_dst);
   b.chunk = reinterpret_cast<int4*>(w + k.chunk);
   b.chunk_base = reinterpret_cast<int64_t*>(w + k.chunk_base);
   b.heavy = reinterpret_cast<int4*>(w + k.heavy);
@@ -483,6 +485,7 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   c->item_cnt = b.item_cnt;
   c->worker = worker;
   c->item_rep = b.item_rep;
+  c->rec_dst = b.rec_dst;
   c->dR = dR;
   c->dL = dL;
   c->chunk = b.chunk;
@@ -519,6 +522,7 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   a.uoff = c->uoff + (int64_t)b * (c->n_users + 1);
   a.rec_j = c->rec_j + c->mb_base[b];
   a.rec_D = c->rec_D + c->mb_base[b];
+  a.rec_dst = c->rec_dst + c->mb_base[b];
   a.item_rep = c->item_rep;
   a.dR = c->dR;
   a.eta = eta;

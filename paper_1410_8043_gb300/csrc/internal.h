@@ -54,6 +54,7 @@ struct SgdArgs {
   const int32_t* uoff;      // [n_users+1] entry offsets of minibatch b (relative)
   const int32_t* rec_j;     // item of each entry of minibatch b
   const float* rec_D;       // value of each entry of minibatch b
+  const int32_t* rec_dst;   // replica row in dR that each entry's item update adds into
   const int32_t* item_rep;  // [M+1] first replica row of each item in dR
   float* dR;                // item delta replicas (all zero between clocks)
   float eta, lambda;
@@ -122,6 +123,7 @@ struct LayoutBuild {
   int32_t* rec_u;
   int32_t* rec_j;
   float* rec_D;
+  int32_t* rec_dst;     // replica row of each entry's item update
   int32_t* uoff;        // [F][n_users+1]
   int64_t* mb_base;     // [F+1]
   int32_t* item_cnt;    // [F][n_items]

@@ -150,6 +150,21 @@ __global__ void item_reps_kernel(const int32_t* __restrict__ item_cnt, int64_t n
   }
 }
 
+// Replica row of every entry's item update: entry t (position within its
+// minibatch) of item j adds into row item_rep[j] + (t mod replicas of j).
+__global__ void dst_kernel(const uint32_t* __restrict__ key, const int64_t* __restrict__ mb_base,
+                           const int32_t* __restrict__ rec_j, const int32_t* __restrict__ item_rep, int64_t n_obs,
+                           int64_t n_users, int32_t* __restrict__ rec_dst) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < n_obs; k += stride) {
+    const int64_t b = (int64_t)key[k] / n_users;
+    const int64_t t = k - mb_base[b];
+    const int32_t j = rec_j[k];
+    const int32_t r0 = item_rep[j], r1 = item_rep[j + 1];
+    rec_dst[k] = r0 + (int32_t)(t & (int64_t)(r1 - r0 - 1));
+  }
+}
+
 int blocks_for(int64_t n) {
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
@@ -273,7 +288,12 @@ cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st) {
   item_reps_kernel<<<blocks_for(b.n_items + 1), 256, 0, st>>>(b.item_cnt, b.n_items, b.F, ireps);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   tb = p.cub_bytes;
-  return cub::DeviceScan::ExclusiveSum(cub_tmp, tb, ireps, b.item_rep, (int)(b.n_items + 1), st);
+  if ((e = cub::DeviceScan::ExclusiveSum(cub_tmp, tb, ireps, b.item_rep, (int)(b.n_items + 1), st)) != cudaSuccess)
+    return e;
+  if (b.n_obs == 0) return cudaSuccess;
+  dst_kernel<<<blocks_for(b.n_obs), 256, 0, st>>>(key_out, b.mb_base, b.rec_j, b.item_rep, b.n_obs, b.n_users,
+                                                  b.rec_dst);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_validate(const LayoutBuild& b, cudaStream_t st) {

@@ -47,21 +47,18 @@ __device__ __forceinline__ float cap_scale(int32_t cap, int32_t n) {
   return (cap > 0 && n > cap) ? (float)cap / (float)n : 1.f;
 }
 
-// Entry t of the minibatch (item, value); zeros past the end.
-__device__ __forceinline__ void load_entry(const SgdArgs& a, int32_t t, int32_t& j, float& d) {
+// Entry t of the minibatch: item, value and the replica row its item update
+// adds into; zeros past the end.
+__device__ __forceinline__ void load_entry(const SgdArgs& a, int32_t t, int32_t& j, float& d, int32_t& dst) {
   if (t < a.n_b) {
     j = __ldg(a.rec_j + t);
     d = __ldg(a.rec_D + t);
+    dst = __ldg(a.rec_dst + t);
   } else {
     j = 0;
     d = 0.f;
+    dst = 0;
   }
-}
-
-// Replica row of item j that entry t adds into.
-__device__ __forceinline__ int32_t replica_row(const SgdArgs& a, int32_t t, int32_t j) {
-  const int32_t r0 = __ldg(a.item_rep + j), r1 = __ldg(a.item_rep + j + 1);
-  return r0 + (t & (r1 - r0 - 1));
 }
 
 // A group's sliding window over the minibatch entries: lane l holds entry
@@ -69,14 +66,13 @@ __device__ __forceinline__ int32_t replica_row(const SgdArgs& a, int32_t t, int3
 template <int G>
 struct Window {
   int32_t W;
-  int32_t cj, cdst, nj;
+  int32_t cj, cdst, nj, ndst;
   float cd, nd;
 
   __device__ __forceinline__ void reload(const SgdArgs& a, int32_t start, int glane) {
     W = start;
-    load_entry(a, W + glane, cj, cd);
-    cdst = replica_row(a, W + glane, cj);
-    load_entry(a, W + G + glane, nj, nd);
+    load_entry(a, W + glane, cj, cd, cdst);
+    load_entry(a, W + G + glane, nj, nd, ndst);
   }
   // Make entry t (>= W) part of cur.
   __device__ __forceinline__ void cover(const SgdArgs& a, int32_t t, int glane) {
@@ -85,74 +81,91 @@ struct Window {
       W += G;
       cj = nj;
       cd = nd;
-      cdst = replica_row(a, W + glane, cj);
-      load_entry(a, W + G + glane, nj, nd);
+      cdst = ndst;
+      load_entry(a, W + G + glane, nj, nd, ndst);
     } else {
       reload(a, t, glane);
     }
   }
 };
 
-// Entries [t0, t0 + nbat) of one row group, all inside the window's cur part
-// and all of one user whose read-version row is Lv.  For each entry:
-// e = D - L.R at the read version; gL += e R - lambda L; the item update
-// e L - lambda R goes (unscaled) into the entry's replica row of dR.
-template <int G, int NV, int B>
-__device__ __forceinline__ void process_batch(const SgdArgs& a, const Window<G>& win, int32_t t0, int32_t nbat,
-                                              const float4 (&Lv)[NV], float4 (&gL)[NV],
-                                              const float4* __restrict__ Rv_base, float4* __restrict__ dR4,
-                                              int glane, unsigned gmask, int32_t K4, float& loss) {
-  const int32_t i0 = t0 - win.W;
-  int32_t jj[B];
-  float4 R[B][NV];
+// U entries (U = 1 or 2) of one row group, sitting in lanes i, i+1, ... of the
+// window's cur part, all of one user whose read-version row is Lv.  For each:
+// e = D - L.R at the read version; gL += e R (process_range adds the
+// -lambda L terms once); the item update e L - lambda R goes (unscaled) into
+// the entry's replica row of dR.  Rq and dRq already point at the lane's first
+// slice (+glane); act[t] marks the slices inside the row (glane + t G < K4).
+template <int G, int NV, int U>
+__device__ __forceinline__ void process_entries(const SgdArgs& a, const Window<G>& win, int32_t i,
+                                                const float4 (&Lv)[NV], float4 (&gL)[NV],
+                                                const float4* __restrict__ Rq, float4* __restrict__ dRq,
+                                                const bool (&act)[NV], unsigned gmask, int32_t K4, float& loss) {
+  float4 R[U][NV];
+  int32_t dst[U];
+  float d[U], part[U];
 #pragma unroll
-  for (int u = 0; u < B; ++u) {
-    jj[u] = __shfl_sync(gmask, win.cj, (i0 + u) & (G - 1), G);
+  for (int u = 0; u < U; ++u) {
+    const float4* row = Rq + __shfl_sync(gmask, win.cj, i + u, G) * K4;
 #pragma unroll
-    for (int t = 0; t < NV; ++t) {
-      const int32_t q = glane + t * G;
-      R[u][t] = (u < nbat && q < K4) ? __ldg(Rv_base + (int64_t)jj[u] * K4 + q) : f4_zero();
-    }
+    for (int t = 0; t < NV; ++t) R[u][t] = act[t] ? __ldg(row + t * G) : f4_zero();
   }
 #pragma unroll
-  for (int u = 0; u < B; ++u) {
-    const float d = __shfl_sync(gmask, win.cd, (i0 + u) & (G - 1), G);
-    const int32_t dst = __shfl_sync(gmask, win.cdst, (i0 + u) & (G - 1), G);
-    if (u < nbat) {
-      float part = 0.f;
+  for (int u = 0; u < U; ++u) {
+    d[u] = __shfl_sync(gmask, win.cd, i + u, G);
+    dst[u] = __shfl_sync(gmask, win.cdst, i + u, G);
+    part[u] = 0.f;
 #pragma unroll
-      for (int t = 0; t < NV; ++t) part += dot4(Lv[t], R[u][t]);
-      const float e = d - group_sum<G>(part, gmask);
-      loss += e * e;
+    for (int t = 0; t < NV; ++t) part[u] += dot4(Lv[t], R[u][t]);
+  }
 #pragma unroll
-      for (int t = 0; t < NV; ++t) {
-        const int32_t q = glane + t * G;
-        if (q < K4) {
-          const float4 r = R[u][t], l = Lv[t];
-          gL[t].x += e * r.x - a.lambda * l.x;
-          gL[t].y += e * r.y - a.lambda * l.y;
-          gL[t].z += e * r.z - a.lambda * l.z;
-          gL[t].w += e * r.w - a.lambda * l.w;
-          red_add_v4(dR4 + (int64_t)dst * K4 + q, make_float4(e * l.x - a.lambda * r.x, e * l.y - a.lambda * r.y,
-                                                              e * l.z - a.lambda * r.z, e * l.w - a.lambda * r.w));
-        }
-      }
+  for (int off = G / 2; off > 0; off >>= 1) {
+#pragma unroll
+    for (int u = 0; u < U; ++u) part[u] += __shfl_xor_sync(gmask, part[u], off, G);
+  }
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    const float e = d[u] - part[u];
+    loss += e * e;
+    float4* out = dRq + dst[u] * K4;
+#pragma unroll
+    for (int t = 0; t < NV; ++t) {
+      const float4 r = R[u][t], l = Lv[t];
+      gL[t].x += e * r.x;
+      gL[t].y += e * r.y;
+      gL[t].z += e * r.z;
+      gL[t].w += e * r.w;
+      red_add_v4_if(out + t * G,
+                    make_float4(e * l.x - a.lambda * r.x, e * l.y - a.lambda * r.y, e * l.z - a.lambda * r.z,
+                                e * l.w - a.lambda * r.w),
+                    act[t]);
     }
   }
 }
 
-// All entries [beg, end) of one user (or chunk), batch by batch.
-template <int G, int NV, int B>
+// All entries [beg, end) of one user (or chunk), two at a time:
+// gL += sum_k (e_k R_j - lambda L_i).
+template <int G, int NV>
 __device__ __forceinline__ void process_range(const SgdArgs& a, Window<G>& win, int32_t beg, int32_t end,
                                               const float4 (&Lv)[NV], float4 (&gL)[NV],
-                                              const float4* __restrict__ Rv_base, float4* __restrict__ dR4,
-                                              int glane, unsigned gmask, int32_t K4, float& loss) {
-  for (int32_t t0 = beg; t0 < end;) {
-    win.cover(a, t0, glane);
-    const int32_t nbat = min(B, min(end - t0, win.W + G - t0));
-    process_batch<G, NV, B>(a, win, t0, nbat, Lv, gL, Rv_base, dR4, glane, gmask, K4, loss);
-    t0 += nbat;
+                                              const float4* __restrict__ Rq, float4* __restrict__ dRq,
+                                              const bool (&act)[NV], int glane, unsigned gmask, int32_t K4,
+                                              float& loss) {
+  int32_t t = beg;
+  while (t < end) {
+    win.cover(a, t, glane);
+    const int32_t lim = min(end, win.W + G);
+#ifdef ESSPT_STEP4
+    for (; t + 4 <= lim; t += 4) process_entries<G, NV, 4>(a, win, t - win.W, Lv, gL, Rq, dRq, act, gmask, K4, loss);
+#endif
+    for (; t + 2 <= lim; t += 2) process_entries<G, NV, 2>(a, win, t - win.W, Lv, gL, Rq, dRq, act, gmask, K4, loss);
+    if (t < lim) {
+      process_entries<G, NV, 1>(a, win, t - win.W, Lv, gL, Rq, dRq, act, gmask, K4, loss);
+      ++t;
+    }
   }
+  const float nl = -(float)(end - beg) * a.lambda;
+#pragma unroll
+  for (int t2 = 0; t2 < NV; ++t2) gL[t2] = f4_axpy(nl, Lv[t2], gL[t2]);
 }
 
 __device__ __forceinline__ float4 f4_add(float4 a, float4 b) {
@@ -196,18 +209,25 @@ __device__ __forceinline__ void flush_loss(double* out, float v, int lane) {
 // and the next window of entries while it computes the current user.
 //   L_i^c = L_i^base + eta s_i sum_k (e_k R_j - lambda L_i)   (written once)
 // Users with more than kHeavy entries are left to the chunk / heavy-merge path.
-template <int G, int NV, int B>
-__global__ void __launch_bounds__(256) sgd_users_kernel(SgdArgs a) {
+#ifndef ESSPT_USERS_MINB
+#define ESSPT_USERS_MINB 3
+#endif
+template <int G, int NV>
+__global__ void __launch_bounds__(256, ESSPT_USERS_MINB) sgd_users_kernel(SgdArgs a) {
   const int lane = threadIdx.x & 31;
   const int glane = lane & (G - 1);
   const int grp = lane / G;
   const unsigned gmask = group_mask<G>(lane);
   const int32_t K4 = a.K >> 2;
   const int64_t slot4 = a.n_rows * K4;
-  float4* ring4 = reinterpret_cast<float4*>(a.ring);
-  float4* out4 = ring4 + (int64_t)a.slot_out * slot4;
-  const float4* base4 = ring4 + (int64_t)a.slot_base * slot4;
-  float4* dR4 = reinterpret_cast<float4*>(a.dR);
+  // Per-lane base pointers: slice t of row r of a table is p[r * K4 + t * G].
+  float4* ringq = reinterpret_cast<float4*>(a.ring) + glane;
+  float4* outq = ringq + (int64_t)a.slot_out * slot4;
+  const float4* baseq = ringq + (int64_t)a.slot_base * slot4;
+  float4* dRq = reinterpret_cast<float4*>(a.dR) + glane;
+  bool act[NV];
+#pragma unroll
+  for (int t = 0; t < NV; ++t) act[t] = glane + t * G < K4;
   const uint64_t pol = policy_evict_first();
   float loss = 0.f;
   const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -237,12 +257,13 @@ __global__ void __launch_bounds__(256) sgd_users_kernel(SgdArgs a) {
     {
       const int32_t n = nend - nbeg;
       nsame = (nvs == a.slot_base) && n > 0;
+      const float4* pv = ringq + (int64_t)nvs * slot4 + g0 * K4;
+      const float4* pb = baseq + g0 * K4;
 #pragma unroll
       for (int t = 0; t < NV; ++t) {
-        const int32_t q = glane + t * G;
-        const bool in = q < K4 && n <= kHeavy;
-        Lvn[t] = (in && n > 0) ? ld_stream(ring4 + (int64_t)nvs * slot4 + g0 * K4 + q, pol) : f4_zero();
-        Lbn[t] = (in && !nsame) ? ld_stream(base4 + g0 * K4 + q, pol) : f4_zero();
+        const bool in = act[t] && n <= kHeavy;
+        Lvn[t] = ld_stream_if(pv + t * G, pol, in && n > 0);
+        Lbn[t] = ld_stream_if(pb + t * G, pol, in && !nsame);
       }
     }
 
@@ -262,12 +283,13 @@ __global__ void __launch_bounds__(256) sgd_users_kernel(SgdArgs a) {
         nend = __shfl_sync(gmask, m_end, t + 1, G);
         const int32_t n = nend - nbeg;
         nsame = (nvs == a.slot_base) && n > 0;
+        const float4* pv = ringq + (int64_t)nvs * slot4 + (u + 1) * K4;
+        const float4* pb = baseq + (u + 1) * K4;
 #pragma unroll
         for (int k = 0; k < NV; ++k) {
-          const int32_t q = glane + k * G;
-          const bool in = q < K4 && n <= kHeavy;
-          Lvn[k] = (in && n > 0) ? ld_stream(ring4 + (int64_t)nvs * slot4 + (u + 1) * K4 + q, pol) : f4_zero();
-          Lbn[k] = (in && !nsame) ? ld_stream(base4 + (u + 1) * K4 + q, pol) : f4_zero();
+          const bool in = act[k] && n <= kHeavy;
+          Lvn[k] = ld_stream_if(pv + k * G, pol, in && n > 0);
+          Lbn[k] = ld_stream_if(pb + k * G, pol, in && !nsame);
         }
       }
       const int32_t n = end - beg;
@@ -276,16 +298,152 @@ __global__ void __launch_bounds__(256) sgd_users_kernel(SgdArgs a) {
 #pragma unroll
       for (int k = 0; k < NV; ++k) gL[k] = f4_zero();
       if (n > 0) {
-        const float4* Rv_base = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4;
-        process_range<G, NV, B>(a, win, beg, end, Lv, gL, Rv_base, dR4, glane, gmask, K4, loss);
+        const float4* Rq = ringq + (int64_t)vs * slot4 + (int64_t)a.n_users * K4;
+        process_range<G, NV>(a, win, beg, end, Lv, gL, Rq, dRq, act, glane, gmask, K4, loss);
       }
       const float sc = a.eta * cap_scale(a.cap, n);
+      float4* po = outq + u * K4;
 #pragma unroll
-      for (int k = 0; k < NV; ++k) {
-        const int32_t q = glane + k * G;
-        if (q < K4) st_stream(out4 + u * K4 + q, f4_axpy(sc, gL[k], same ? Lv[k] : Lb[k]), pol);
+      for (int k = 0; k < NV; ++k) st_stream_if(po + k * G, f4_axpy(sc, gL[k], same ? Lv[k] : Lb[k]), pol, act[k]);
+    }
+  }
+  flush_loss(a.sq_loss, glane == 0 ? loss : 0.f, lane);
+}
+
+// Rows of 68..128 values (17..32 float4 slices): a group of 8 lanes holds
+// one row, 4 slices per lane (slice q = glane + 8k), and the warp's 4 groups
+// take 4 entries of the same user per step, so one 3-level reduction serves
+// 4 dot products.  The user's rows at the read and base versions are staged
+// in shared memory one user ahead by cp.async.  At the user's end a
+// reduce-scatter over the 4 groups leaves slice glane + 8 grp of the summed
+// user update on each lane, which writes L_i^c for that slice.
+#ifndef ESSPT_USERS4_MINB
+#define ESSPT_USERS4_MINB 3
+#endif
+__global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdArgs a) {
+  constexpr int NV = 4;
+  __shared__ __align__(16) float4 stage[8][2][2][32];  // [warp][buffer][read row, base row][slice]
+  const int lane = threadIdx.x & 31;
+  const int wib = threadIdx.x >> 5;
+  const int glane = lane & 7;
+  const int grp = lane >> 3;
+  const unsigned gmask = group_mask<8>(lane);
+  const int32_t K4 = a.K >> 2;
+  const int64_t slot4 = a.n_rows * K4;
+  float4* ring4 = reinterpret_cast<float4*>(a.ring);
+  float4* outq = ring4 + (int64_t)a.slot_out * slot4;
+  const float4* base4 = ring4 + (int64_t)a.slot_base * slot4;
+  float4* dRq = reinterpret_cast<float4*>(a.dR) + glane;
+  bool act[NV];
+#pragma unroll
+  for (int k = 0; k < NV; ++k) act[k] = glane + 8 * k < K4;
+  const int my_q = glane + 8 * grp;  // the slice this lane writes
+  const bool my_act = my_q < K4;
+  const uint64_t pol = policy_evict_first();
+  float loss = 0.f;
+  const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+
+  for (int64_t u0 = warp_id * 32; u0 < a.n_users; u0 += nwarps * 32) {
+    const int64_t uu = u0 + lane;
+    int32_t m_beg = 0, m_end = 0, m_vs = 0;
+    if (uu < a.n_users) {
+      m_beg = __ldg(a.uoff + uu);
+      m_end = __ldg(a.uoff + uu + 1);
+      m_vs = __ldg(a.v + __ldg(a.worker + uu)) % a.nslots;
+    }
+    const int32_t nusers = (int32_t)min((int64_t)32, (int64_t)a.n_users - u0);
+    Window<32> win;
+    win.reload(a, __shfl_sync(0xffffffffu, m_beg, 0), lane);
+
+    // Stage user t's rows into buffer b: lane l copies slice l of the read
+    // row (if it has entries) and of the base row (if it differs or is the
+    // only row needed).
+    auto stage_user = [&](int32_t t, int b) {
+      const int32_t vs = __shfl_sync(0xffffffffu, m_vs, t);
+      const int32_t n = __shfl_sync(0xffffffffu, m_end, t) - __shfl_sync(0xffffffffu, m_beg, t);
+      const bool same = vs == a.slot_base && n > 0;
+      const bool in = lane < K4 && n <= kHeavy;
+      const float4* pv = ring4 + (int64_t)vs * slot4 + (u0 + t) * K4 + (lane < K4 ? lane : 0);
+      const float4* pb = base4 + (u0 + t) * K4 + (lane < K4 ? lane : 0);
+      cp_async16(&stage[wib][b][0][lane], pv, in && n > 0);
+      cp_async16(&stage[wib][b][1][lane], pb, in && !same);
+      cp_async_commit();
+    };
+    stage_user(0, 0);
+
+    for (int32_t t = 0; t < nusers; ++t) {
+      const int b = t & 1;
+      cp_async_wait_all();
+      __syncwarp();
+      if (t + 1 < nusers) stage_user(t + 1, b ^ 1);
+      const int32_t vs = __shfl_sync(0xffffffffu, m_vs, t);
+      const int32_t beg = __shfl_sync(0xffffffffu, m_beg, t);
+      const int32_t end = __shfl_sync(0xffffffffu, m_end, t);
+      const int32_t n = end - beg;
+      if (n > kHeavy) continue;
+      const float4* Lv_s = &stage[wib][b][0][glane];
+      const float4* Rq = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4 + glane;
+      float4 gL[NV];
+#pragma unroll
+      for (int k = 0; k < NV; ++k) gL[k] = f4_zero();
+      for (int32_t tt = beg; tt < end;) {
+        win.cover(a, tt, lane);
+        const int32_t cnt = min(4, min(end - tt, win.W + 32 - tt));
+        const bool valid = grp < cnt;
+        const int src = min(tt - win.W + grp, 31);
+        const int32_t j = __shfl_sync(0xffffffffu, win.cj, src);
+        const float d = __shfl_sync(0xffffffffu, win.cd, src);
+        const int32_t dst = __shfl_sync(0xffffffffu, win.cdst, src);
+        const float4* row = Rq + j * K4;
+        float4 R[NV];
+#pragma unroll
+        for (int k = 0; k < NV; ++k) R[k] = (act[k] && valid) ? __ldg(row + 8 * k) : f4_zero();
+        float part = 0.f;
+#pragma unroll
+        for (int k = 0; k < NV; ++k) part += dot4(Lv_s[8 * k], R[k]);
+#pragma unroll
+        for (int off = 4; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
+        const float e = valid ? d - part : 0.f;
+        loss += e * e;
+        float4* out = dRq + dst * K4;
+#pragma unroll
+        for (int k = 0; k < NV; ++k) {
+          const float4 r = R[k], l = Lv_s[8 * k];
+          gL[k].x += e * r.x;
+          gL[k].y += e * r.y;
+          gL[k].z += e * r.z;
+          gL[k].w += e * r.w;
+          red_add_v4_if(out + 8 * k,
+                        make_float4(e * l.x - a.lambda * r.x, e * l.y - a.lambda * r.y, e * l.z - a.lambda * r.z,
+                                    e * l.w - a.lambda * r.w),
+                        act[k] && valid);
+        }
+        tt += cnt;
+      }
+      // Reduce-scatter over the groups: group g keeps slice set k = g.
+      {
+        const bool hi = grp >= 2;
+        float4 k0 = hi ? gL[2] : gL[0], k1 = hi ? gL[3] : gL[1];
+        const float4 s0 = hi ? gL[0] : gL[2], s1 = hi ? gL[1] : gL[3];
+        k0 = f4_add(k0, make_float4(__shfl_xor_sync(0xffffffffu, s0.x, 16), __shfl_xor_sync(0xffffffffu, s0.y, 16),
+                                    __shfl_xor_sync(0xffffffffu, s0.z, 16), __shfl_xor_sync(0xffffffffu, s0.w, 16)));
+        k1 = f4_add(k1, make_float4(__shfl_xor_sync(0xffffffffu, s1.x, 16), __shfl_xor_sync(0xffffffffu, s1.y, 16),
+                                    __shfl_xor_sync(0xffffffffu, s1.z, 16), __shfl_xor_sync(0xffffffffu, s1.w, 16)));
+        const bool odd = grp & 1;
+        float4 keep = odd ? k1 : k0;
+        const float4 snd = odd ? k0 : k1;
+        keep = f4_add(keep, make_float4(__shfl_xor_sync(0xffffffffu, snd.x, 8), __shfl_xor_sync(0xffffffffu, snd.y, 8),
+                                        __shfl_xor_sync(0xffffffffu, snd.z, 8), __shfl_xor_sync(0xffffffffu, snd.w, 8)));
+        const bool same = vs == a.slot_base && n > 0;
+        const float4 lv = stage[wib][b][0][my_q];
+        const float4 lb = stage[wib][b][same ? 0 : 1][my_q];
+        const float sc = a.eta * cap_scale(a.cap, n);
+        const float4 g = f4_axpy(-(float)n * a.lambda, lv, keep);
+        st_stream_if(outq + (u0 + t) * K4 + my_q, f4_axpy(sc, g, lb), pol, my_act);
       }
     }
+    __syncwarp();
   }
   flush_loss(a.sq_loss, glane == 0 ? loss : 0.f, lane);
 }
@@ -293,7 +451,7 @@ __global__ void __launch_bounds__(256) sgd_users_kernel(SgdArgs a) {
 // Chunks of at most kChunk entries of users with more than kHeavy entries:
 // the chunk's partial user update sum (e R - lambda L) goes, unscaled, into
 // one of its user's replica rows of dL; item updates as in the user kernel.
-template <int G, int NV, int B>
+template <int G, int NV>
 __global__ void __launch_bounds__(256) sgd_chunks_kernel(ChunkArgs c) {
   const SgdArgs& a = c.a;
   const int lane = threadIdx.x & 31;
@@ -304,6 +462,9 @@ __global__ void __launch_bounds__(256) sgd_chunks_kernel(ChunkArgs c) {
   const float4* ring4 = reinterpret_cast<const float4*>(a.ring);
   float4* dR4 = reinterpret_cast<float4*>(a.dR);
   float4* dL4 = reinterpret_cast<float4*>(c.dL);
+  bool act[NV];
+#pragma unroll
+  for (int t = 0; t < NV; ++t) act[t] = glane + t * G < K4;
   float loss = 0.f;
   const int64_t first = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * (32 / G);
   const int64_t step = (((int64_t)gridDim.x * blockDim.x) >> 5) * (32 / G);
@@ -322,8 +483,8 @@ __global__ void __launch_bounds__(256) sgd_chunks_kernel(ChunkArgs c) {
       }
       Window<G> win;
       win.reload(a, ch.y, glane);
-      const float4* Rv_base = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4;
-      process_range<G, NV, B>(a, win, ch.y, ch.z, Lv, gL, Rv_base, dR4, glane, gmask, K4, loss);
+      const float4* Rq = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4 + glane;
+      process_range<G, NV>(a, win, ch.y, ch.z, Lv, gL, Rq, dR4 + glane, act, glane, gmask, K4, loss);
 #pragma unroll
       for (int t = 0; t < NV; ++t) {
         const int32_t q = glane + t * G;
@@ -400,13 +561,15 @@ int grid_for(int64_t work_items, int64_t per_block, int max_per_sm) {
   return (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sm_count() * max_per_sm));
 }
 
-constexpr int kBatchEntries = 4;
-
 template <int G, int NV>
 struct UsersF {
+  static cudaError_t run4(const SgdArgs& a, cudaStream_t st) {
+    sgd_users4_kernel<<<grid_for(a.n_users, 256, 8), 256, 0, st>>>(a);
+    return cudaGetLastError();
+  }
   static cudaError_t run(const SgdArgs& a, cudaStream_t st) {
     // 8 warps per block, 32 users per warp
-    sgd_users_kernel<G, NV, kBatchEntries><<<grid_for(a.n_users, 256, 8), 256, 0, st>>>(a);
+    sgd_users_kernel<G, NV><<<grid_for(a.n_users, 256, 8), 256, 0, st>>>(a);
     return cudaGetLastError();
   }
 };
@@ -414,7 +577,7 @@ template <int G, int NV>
 struct ChunksF {
   static cudaError_t run(const ChunkArgs& c, cudaStream_t st) {
     if (c.n_chunks <= 0) return cudaSuccess;
-    sgd_chunks_kernel<G, NV, kBatchEntries><<<grid_for(c.n_chunks, 256 / G, 8), 256, 0, st>>>(c);
+    sgd_chunks_kernel<G, NV><<<grid_for(c.n_chunks, 256 / G, 8), 256, 0, st>>>(c);
     return cudaGetLastError();
   }
 };
@@ -429,7 +592,11 @@ cudaError_t dispatch_k(int32_t K, const Arg& a, cudaStream_t st) {
   if (K4 <= 4) return F<4, 1>::run(a, st);
   if (K4 <= 8) return F<8, 1>::run(a, st);
   if (K4 <= 16) return F<16, 1>::run(a, st);
+#ifdef ESSPT_WIDE_ROWS
+  if (K4 <= 32) return F<16, 2>::run(a, st);
+#else
   if (K4 <= 32) return F<32, 1>::run(a, st);
+#endif
   if (K4 <= 64) return F<32, 2>::run(a, st);
   if (K4 <= 96) return F<32, 3>::run(a, st);
   return F<32, 4>::run(a, st);
@@ -437,7 +604,12 @@ cudaError_t dispatch_k(int32_t K, const Arg& a, cudaStream_t st) {
 
 }  // namespace
 
-cudaError_t launch_sgd_users(const SgdArgs& a, cudaStream_t st) { return dispatch_k<UsersF>(a.K, a, st); }
+cudaError_t launch_sgd_users(const SgdArgs& a, cudaStream_t st) {
+#ifndef ESSPT_NO_USERS4
+  if (a.K > 64 && a.K <= 128) return UsersF<8, 4>::run4(a, st);
+#endif
+  return dispatch_k<UsersF>(a.K, a, st);
+}
 cudaError_t launch_sgd_chunks(const ChunkArgs& c, cudaStream_t st) { return dispatch_k<ChunksF>(c.a.K, c, st); }
 
 cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st) {

@@ -43,6 +43,45 @@ __device__ __forceinline__ void st_stream(float4* p, float4 v, uint64_t pol) {
                : "memory");
 }
 
+// Predicated forms: the access happens only when `pred` is true, without a
+// branch around the asm (loads give zeros when it is false).
+__device__ __forceinline__ float4 ld_stream_if(const float4* p, uint64_t pol, bool pred) {
+  float4 r;
+  asm volatile(
+      "{\n .reg .pred q;\n setp.ne.b32 q, %5, 0;\n mov.f32 %0, 0f00000000;\n mov.f32 %1, 0f00000000;\n"
+      " mov.f32 %2, 0f00000000;\n mov.f32 %3, 0f00000000;\n"
+      " @q ld.global.L1::no_allocate.L2::cache_hint.v4.f32 {%0,%1,%2,%3}, [%4], %6;\n}"
+      : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w)
+      : "l"(p), "r"((int)pred), "l"(pol));
+  return r;
+}
+
+__device__ __forceinline__ void st_stream_if(float4* p, float4 v, uint64_t pol, bool pred) {
+  asm volatile(
+      "{\n .reg .pred q;\n setp.ne.b32 q, %5, 0;\n"
+      " @q st.global.L1::no_allocate.L2::cache_hint.v4.f32 [%0], {%1,%2,%3,%4}, %6;\n}"
+      :
+      : "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"((int)pred), "l"(pol)
+      : "memory");
+}
+
+__device__ __forceinline__ void red_add_v4_if(float4* p, float4 v, bool pred) {
+  asm volatile(
+      "{\n .reg .pred q;\n setp.ne.b32 q, %5, 0;\n @q red.global.add.v4.f32 [%0], {%1,%2,%3,%4};\n}"
+      :
+      : "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"((int)pred)
+      : "memory");
+}
+
+// 16-byte asynchronous global -> shared copy (bypassing L1); when `pred` is
+// false the 16 shared bytes are zero-filled and nothing is read.
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, bool pred) {
+  const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(s), "l"(gmem), "r"(pred ? 16 : 0) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 // out[0..3] += v, performed at L2 (no return value).
 __device__ __forceinline__ void red_add_v4(float4* p, float4 v) {
   asm volatile("red.global.add.v4.f32 [%0], {%1,%2,%3,%4};"
