@@ -31,6 +31,28 @@ METRIC = "SGD ratings/sec per clock on 1 GB300; achieved HBM GB/s vs peak"
 UNIT = "ratings/s"
 
 
+def _profiled_traffic(kernel: str):
+    """DRAM bytes per launch of `kernel` from its committed ncu summary under
+    profiles/, or None when the kernel source changed since the capture."""
+    import glob
+    import hashlib
+
+    src = os.path.join(ROOT, "paper_1410_8043_gb300", "csrc", "mf_kernels.cu")
+    try:
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    except OSError:
+        return None
+    for path in glob.glob(os.path.join(ROOT, "profiles", f"{kernel}_*.md")):
+        fields = {}
+        for line in open(path):
+            if ":" in line and not line.startswith(("|", "#", " ", "`")):
+                k, _, v = line.partition(":")
+                fields[k.strip()] = v.strip()
+        if fields.get("kernel_source_sha256_16") == digest and "traffic_bytes_per_launch" in fields:
+            return float(fields["traffic_bytes_per_launch"])
+    return None
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -287,6 +309,7 @@ def run_gpu(args, w):
     floor_avg = statistics.mean(floors)
     peak, peak_kind = _peaks()
     achieved = floor_avg / kern_avg_s / 1e9
+    kernel = "sgd_users4_kernel" if 64 < w.K <= 128 else "sgd_users_kernel"
     n_avg = ratings / K
     B_model = 12 + 16 * w.K + 8 * w.K * (w.n_users + w.n_items) / n_avg
     out = {
@@ -312,13 +335,13 @@ def run_gpu(args, w):
         },
         "roofline": {
             "bound": "hbm",
-            "kernel": "sgd_users_kernel (+ sgd_chunks_kernel when present)",
+            "kernel": kernel + " (+ sgd_chunks_kernel / heavy_merge_kernel when some user is heavy)",
             "achieved": achieved,
             "peak": peak,
             "peak_kind": peak_kind,
             "unit": "GB/s",
             "frac": achieved / peak,
-            "traffic": None,
+            "traffic": _profiled_traffic(kernel),
             "algorithmic_bytes_per_launch": floor_avg,
             "kernel_ms": statistics.mean(kern_ms),
             "modelled_bytes_per_rating": B_model,
