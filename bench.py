@@ -177,10 +177,13 @@ class FloorModel:
         self.n = np.zeros(w.F, np.int64)
         self.users_of = np.zeros((w.F, P), np.int64)
         self.items_of = []
+        self.heavy = np.zeros(w.F, bool)
         for b in range(w.F):
             idx = np.flatnonzero(mb == b)
             ui, jj = data.i[idx], data.j[idx]
             self.n[b] = idx.size
+            # users with more than 96 entries go through two extra kernels
+            self.heavy[b] = idx.size > 0 and np.bincount(ui).max() > 96
             has = np.zeros(w.n_users, bool)
             has[ui] = True
             self.users_of[b] = np.bincount(wp[has], minlength=P)
@@ -226,6 +229,7 @@ def run_gpu(args, w):
     K, W = args.steps, args.warmup
     # Accounting pass (untimed): read versions of every clock -> floor bytes.
     floors, counts = [], []
+    stale = np.zeros(w.s + 1, np.int64)
     for c in range(1, W + K + 1):
         v, clk = t.read_schedule()
         assert clk == c
@@ -233,6 +237,7 @@ def run_gpu(args, w):
             fb, n = model.bytes(c, v)
             floors.append(fb)
             counts.append(n)
+            stale += np.bincount(c - 1 - v, minlength=w.s + 1)[: w.s + 1]
         t.mf_sgd_clock(w.eta, w.lam, w.cap)
     t.poll()
     sq0, pen0 = None, None
@@ -348,9 +353,15 @@ def run_gpu(args, w):
             "modelled_GBps": n_avg * B_model / kern_avg_s / 1e9,
         },
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d // K, "d2h_bytes_per_step": d2h // K},
-        "gpu_launches": K * (3 if t.n_users else 2),
+        # per clock: the SGD kernel and the item merge (which also computes the
+        # next schedule), plus the chunk and heavy-merge kernels on minibatches
+        # with heavy users
+        "gpu_launches": int(sum(2 + 2 * model.heavy[(c - 1) % w.F] for c in range(W + 1, W + K + 1))),
         "clocks": clocks,
         "objective": {"clock": c_final, "sq_loss": sq, "penalised": pen},
+        # Fig. 1 (left) quantity: clock differential v_p(c) - c of every read in
+        # the timed clocks (-1 = freshest version; BSP always gives -1).
+        "clock_differential": {str(-1 - k): float(stale[k] / stale.sum()) for k in range(w.s + 1)},
         "setup_s": {"generate": gen_s},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -114,19 +114,10 @@ esspt_status need_schedule(esspt_ctx* c) {
 }
 
 // Compute v_p(clock) on the device (or only check it, for ESSPT_EXTERNAL).
+ScheduleArgs schedule_args(const esspt_ctx* c, int32_t clock);
+
 esspt_status run_schedule(esspt_ctx* c) {
-  ScheduleArgs a{};
-  a.v = c->v;
-  a.status = c->status;
-  a.thr = c->thr;
-  a.P = c->P;
-  a.c = c->clock;
-  a.s = c->s;
-  a.model = c->cfg.model;
-  a.phased = c->cfg.phased;
-  a.dmax = c->dmax;
-  a.seed = c->cfg.seed;
-  ESSPT_CUDA(c, launch_schedule(a, c->st));
+  ESSPT_CUDA(c, launch_schedule(schedule_args(c, c->clock), c->st));
   return ESSPT_OK;
 }
 
@@ -138,13 +129,29 @@ esspt_status ensure_acc(esspt_ctx* c) {
   return ESSPT_OK;
 }
 
-// Version `clock` is final: advance and schedule the next clock.
-esspt_status advance(esspt_ctx* c) {
+// Version `clock` is final: advance and schedule the next clock (unless a
+// kernel of the clock already did, `scheduled`).
+esspt_status advance(esspt_ctx* c, bool scheduled = false) {
   c->clock += 1;
   c->acc_ready = false;
   c->sched_set = false;
-  if (c->cfg.model == ESSPT_EXTERNAL) return ESSPT_OK;
+  if (c->cfg.model == ESSPT_EXTERNAL || scheduled) return ESSPT_OK;
   return run_schedule(c);
+}
+
+ScheduleArgs schedule_args(const esspt_ctx* c, int32_t clock) {
+  ScheduleArgs a{};
+  a.v = c->v;
+  a.status = c->status;
+  a.thr = c->thr;
+  a.P = c->P;
+  a.c = clock;
+  a.s = c->s;
+  a.model = c->cfg.model;
+  a.phased = c->cfg.phased;
+  a.dmax = c->dmax;
+  a.seed = c->cfg.seed;
+  return a;
 }
 
 bool is_host_ptr(const void* p) {
@@ -570,9 +577,11 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   m.item_cnt = c->item_cnt + (int64_t)b * c->n_items;
   m.eta = eta;
   m.cap = cap;
+  m.do_schedule = c->cfg.model != ESSPT_EXTERNAL;
+  m.sched = schedule_args(c, c->clock + 1);
   ESSPT_CUDA(c, launch_item_merge(m, c->st));
   c->acc_ready = true;
-  return advance(c);
+  return advance(c, m.do_schedule != 0);
 }
 
 esspt_status esspt_mf_objective(esspt_ctx* c, int32_t version, float lambda, double* d_scratch, double* h_sq,

@@ -27,9 +27,15 @@ constexpr int32_t kChunk = 64;
 // (largest minibatch count, rounded up to a power of two); a heavy user one
 // per kUserRep chunks.  Replicas spread the fp32 reductions of popular rows
 // over many L2 addresses and keep each partial sum short.
-constexpr int32_t kItemRep = 2048;
+#ifndef ESSPT_ITEM_REP
+#define ESSPT_ITEM_REP 2048
+#endif
+constexpr int32_t kItemRep = ESSPT_ITEM_REP;
 constexpr int32_t kUserRep = 64;
-constexpr int32_t kMaxRep = 512;
+#ifndef ESSPT_MAX_REP
+#define ESSPT_MAX_REP 64
+#endif
+constexpr int32_t kMaxRep = ESSPT_MAX_REP;
 
 struct ScheduleArgs {
   int32_t* v;              // [P] read versions (in: v(c-1), out: v(c))
@@ -92,6 +98,8 @@ struct ItemMergeArgs {
   const int32_t* item_cnt;  // [M] entries per item in minibatch b
   float eta;
   int32_t cap;
+  int32_t do_schedule;      // also compute the next clock's read versions
+  ScheduleArgs sched;
 };
 
 // Launchers (return the launch error, if any).

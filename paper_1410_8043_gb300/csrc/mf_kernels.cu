@@ -12,6 +12,7 @@
 
 #include "internal.h"
 #include "ptx.cuh"
+#include "schedule.cuh"
 
 namespace esspt {
 
@@ -522,24 +523,27 @@ __global__ void __launch_bounds__(256) heavy_merge_kernel(HeavyMergeArgs a) {
 
 // Clock() merge of the item rows (Sec. 2.1 additive updates, Sec. 4 server
 // clock): R^c_j = R^base_j + eta s_j sum of j's replica rows; replicas
-// cleared.  One warp per item.
+// cleared.  One thread per (item, float4 slice).  With do_schedule the first
+// P threads also compute the next clock's read versions (the SGD kernels of
+// this clock, the only readers of v, have finished).
 __global__ void __launch_bounds__(256) item_merge_kernel(ItemMergeArgs a) {
-  const int lane = threadIdx.x & 31;
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t nth = (int64_t)gridDim.x * blockDim.x;
+  if (a.do_schedule)
+    for (int64_t p = tid; p < a.sched.P; p += nth) schedule_worker(a.sched, (int32_t)p);
   const int32_t K4 = a.K >> 2;
   const int64_t slot4 = a.n_rows * K4;
   float4* ring4 = reinterpret_cast<float4*>(a.ring);
   float4* dR4 = reinterpret_cast<float4*>(a.dR);
-  for (int64_t j = warp; j < a.n_items; j += nwarps) {
+  const int64_t total = (int64_t)a.n_items * K4;
+  for (int64_t x = tid; x < total; x += nth) {
+    const int64_t j = x / K4;
+    const int32_t q = (int32_t)(x - j * K4);
     const int32_t r0 = __ldg(a.item_rep + j), r1 = __ldg(a.item_rep + j + 1);
     const float sc = a.eta * cap_scale(a.cap, __ldg(a.item_cnt + j));
-    const int64_t row = (int64_t)a.n_users + j;
-    for (int32_t q = lane; q < K4; q += 32) {
-      const float4 acc = sum_and_clear(dR4 + (int64_t)r0 * K4 + q, r1 - r0, K4);
-      const float4 b = ring4[(int64_t)a.slot_base * slot4 + row * K4 + q];
-      ring4[(int64_t)a.slot_out * slot4 + row * K4 + q] = f4_axpy(sc, acc, b);
-    }
+    const float4 acc = sum_and_clear(dR4 + (int64_t)r0 * K4 + q, r1 - r0, K4);
+    const int64_t row = ((int64_t)a.n_users + j) * K4 + q;
+    ring4[(int64_t)a.slot_out * slot4 + row] = f4_axpy(sc, acc, ring4[(int64_t)a.slot_base * slot4 + row]);
   }
 }
 
@@ -619,8 +623,9 @@ cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st) {
 }
 
 cudaError_t launch_item_merge(const ItemMergeArgs& a, cudaStream_t st) {
-  if (a.n_items <= 0) return cudaSuccess;
-  item_merge_kernel<<<grid_for(a.n_items, 8, 16), 256, 0, st>>>(a);
+  const int64_t work = std::max<int64_t>((int64_t)a.n_items * (a.K >> 2), a.do_schedule ? a.sched.P : 0);
+  if (work <= 0) return cudaSuccess;
+  item_merge_kernel<<<grid_for(work, 256, 16), 256, 0, st>>>(a);
   return cudaGetLastError();
 }
 
