@@ -596,8 +596,10 @@ cudaError_t dispatch_k(int32_t K, const Arg& a, cudaStream_t st) {
   if (K4 <= 4) return F<4, 1>::run(a, st);
   if (K4 <= 8) return F<8, 1>::run(a, st);
   if (K4 <= 16) return F<16, 1>::run(a, st);
-#ifdef ESSPT_WIDE_ROWS
+#if defined(ESSPT_WIDE_ROWS)
   if (K4 <= 32) return F<16, 2>::run(a, st);
+#elif defined(ESSPT_QUAD_ROWS)
+  if (K4 <= 32) return F<8, 4>::run(a, st);
 #else
   if (K4 <= 32) return F<32, 1>::run(a, st);
 #endif
