@@ -193,7 +193,7 @@ MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int
   k.mb_base = take(sizeof(int64_t) * (F + 1));
   k.item_cnt = take(sizeof(int32_t) * (size_t)F * n_items);
   k.item_rep = take(sizeof(int32_t) * (n_items + 1));
-  k.dR = take(sizeof(float) * (size_t)k.dR_rows * K);
+  k.dR = take(sizeof(float4) * (size_t)k.dR_rows * dR_stride4(K));
   k.worker = take(sizeof(int32_t) * n_users);
   k.chunk = take(sizeof(int4) * k.max_chunks);
   k.chunk_base = take(sizeof(int64_t) * (F + 1));
@@ -465,7 +465,7 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   ESSPT_CUDA(c, cudaMemcpyAsync(worker, d_worker, sizeof(int32_t) * n_users, cudaMemcpyDeviceToDevice, c->st));
   float* dR = reinterpret_cast<float*>(w + k.dR);
   float* dL = reinterpret_cast<float*>(w + k.dL);
-  ESSPT_CUDA(c, cudaMemsetAsync(dR, 0, sizeof(float) * (size_t)k.dR_rows * c->K, c->st));
+  ESSPT_CUDA(c, cudaMemsetAsync(dR, 0, sizeof(float4) * (size_t)k.dR_rows * dR_stride4(c->K), c->st));
   ESSPT_CUDA(c, cudaMemsetAsync(dL, 0, sizeof(float) * (size_t)k.dL_rows * c->K, c->st));
   ESSPT_CUDA(c, cudaMemsetAsync(b.rec_u + n_obs, 0, 16, c->st));
   ESSPT_CUDA(c, cudaMemsetAsync(b.rec_j + n_obs, 0, 16, c->st));
@@ -532,6 +532,7 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   a.rec_dst = c->rec_dst + c->mb_base[b];
   a.item_rep = c->item_rep;
   a.dR = c->dR;
+  a.dR_ld = dR_stride4(c->K);
   a.eta = eta;
   a.lambda = lambda;
   a.cap = cap;
@@ -574,6 +575,7 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   m.slot_out = slot_out;
   m.item_rep = c->item_rep;
   m.dR = c->dR;
+  m.dR_ld = dR_stride4(c->K);
   m.item_cnt = c->item_cnt + (int64_t)b * c->n_items;
   m.eta = eta;
   m.cap = cap;

@@ -37,6 +37,10 @@ constexpr int32_t kUserRep = 64;
 #endif
 constexpr int32_t kMaxRep = ESSPT_MAX_REP;
 
+// Row stride (in float4) of the item delta replicas: K rounded up to a whole
+// number of 32-byte sectors, so that a row's reductions touch the fewest sectors.
+inline int32_t dR_stride4(int32_t K) { return ((K + 7) / 8) * 2; }
+
 struct ScheduleArgs {
   int32_t* v;              // [P] read versions (in: v(c-1), out: v(c))
   uint32_t* status;        // latched error bits
@@ -63,6 +67,7 @@ struct SgdArgs {
   const int32_t* rec_dst;   // replica row in dR that each entry's item update adds into
   const int32_t* item_rep;  // [M+1] first replica row of each item in dR
   float* dR;                // item delta replicas (all zero between clocks)
+  int32_t dR_ld;            // float4 per dR row (K rounded up to whole 32-byte sectors)
   float eta, lambda;
   int32_t cap;
   double* sq_loss;          // optional
@@ -95,6 +100,7 @@ struct ItemMergeArgs {
   int32_t K, n_users, n_items, slot_base, slot_out;
   const int32_t* item_rep;
   float* dR;
+  int32_t dR_ld;
   const int32_t* item_cnt;  // [M] entries per item in minibatch b
   float eta;
   int32_t cap;

@@ -127,7 +127,7 @@ __device__ __forceinline__ void process_entries(const SgdArgs& a, const Window<G
   for (int u = 0; u < U; ++u) {
     const float e = d[u] - part[u];
     loss += e * e;
-    float4* out = dRq + dst[u] * K4;
+    float4* out = dRq + dst[u] * a.dR_ld;
 #pragma unroll
     for (int t = 0; t < NV; ++t) {
       const float4 r = R[u][t], l = Lv[t];
@@ -407,7 +407,7 @@ __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdA
         for (int off = 4; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
         const float e = valid ? d - part : 0.f;
         loss += e * e;
-        float4* out = dRq + dst * K4;
+        float4* out = dRq + dst * a.dR_ld;
 #pragma unroll
         for (int k = 0; k < NV; ++k) {
           const float4 r = R[k], l = Lv_s[8 * k];
@@ -541,7 +541,7 @@ __global__ void __launch_bounds__(256) item_merge_kernel(ItemMergeArgs a) {
     const int32_t q = (int32_t)(x - j * K4);
     const int32_t r0 = __ldg(a.item_rep + j), r1 = __ldg(a.item_rep + j + 1);
     const float sc = a.eta * cap_scale(a.cap, __ldg(a.item_cnt + j));
-    const float4 acc = sum_and_clear(dR4 + (int64_t)r0 * K4 + q, r1 - r0, K4);
+    const float4 acc = sum_and_clear(dR4 + (int64_t)r0 * a.dR_ld + q, r1 - r0, a.dR_ld);
     const int64_t row = ((int64_t)a.n_users + j) * K4 + q;
     ring4[(int64_t)a.slot_out * slot4 + row] = f4_axpy(sc, acc, ring4[(int64_t)a.slot_base * slot4 + row]);
   }

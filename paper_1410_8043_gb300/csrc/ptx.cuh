@@ -65,12 +65,11 @@ __device__ __forceinline__ void st_stream_if(float4* p, float4 v, uint64_t pol, 
       : "memory");
 }
 
+// out[0..3] += v when `pred`, performed at L2.  The return value of the
+// vector atomicAdd (sm_90 and later) is unused, so it issues as a reduction;
+// the compiler predicates it without a branch.
 __device__ __forceinline__ void red_add_v4_if(float4* p, float4 v, bool pred) {
-  asm volatile(
-      "{\n .reg .pred q;\n setp.ne.b32 q, %5, 0;\n @q red.global.add.v4.f32 [%0], {%1,%2,%3,%4};\n}"
-      :
-      : "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"((int)pred)
-      : "memory");
+  if (pred) atomicAdd(p, v);
 }
 
 // 16-byte asynchronous global -> shared copy (bypassing L1); when `pred` is
@@ -83,12 +82,7 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 // out[0..3] += v, performed at L2 (no return value).
-__device__ __forceinline__ void red_add_v4(float4* p, float4 v) {
-  asm volatile("red.global.add.v4.f32 [%0], {%1,%2,%3,%4};"
-               :
-               : "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
-               : "memory");
-}
+__device__ __forceinline__ void red_add_v4(float4* p, float4 v) { atomicAdd(p, v); }
 
 // SplitMix64 (Steele, Lea and Flood, OOPSLA 2014): output n of the sequence
 // whose state starts at s0 is mix64(s0 + n * 0x9E3779B97F4A7C15).
