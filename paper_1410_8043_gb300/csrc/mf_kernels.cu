@@ -52,9 +52,10 @@ __device__ __forceinline__ float cap_scale(int32_t cap, int32_t n) {
 // adds into; zeros past the end.
 __device__ __forceinline__ void load_entry(const SgdArgs& a, int32_t t, int32_t& j, float& d, int32_t& dst) {
   if (t < a.n_b) {
-    j = __ldg(a.rec_j + t);
-    d = __ldg(a.rec_D + t);
-    dst = __ldg(a.rec_dst + t);
+    const uint64_t pol = policy_evict_first();
+    j = ld_stream_i32(a.rec_j + t, pol);
+    d = ld_stream_f32(a.rec_D + t, pol);
+    dst = ld_stream_i32(a.rec_dst + t, pol);
   } else {
     j = 0;
     d = 0.f;
@@ -367,8 +368,8 @@ __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdA
       const bool in = lane < K4 && n <= kHeavy;
       const float4* pv = ring4 + (int64_t)vs * slot4 + (u0 + t) * K4 + (lane < K4 ? lane : 0);
       const float4* pb = base4 + (u0 + t) * K4 + (lane < K4 ? lane : 0);
-      cp_async16(&stage[wib][b][0][lane], pv, in && n > 0);
-      cp_async16(&stage[wib][b][1][lane], pb, in && !same);
+      cp_async16_hint(&stage[wib][b][0][lane], pv, in && n > 0, pol);
+      cp_async16_hint(&stage[wib][b][1][lane], pb, in && !same, pol);
       cp_async_commit();
     };
     stage_user(0, 0);
