@@ -319,9 +319,20 @@ __global__ void __launch_bounds__(256, ESSPT_USERS_MINB) sgd_users_kernel(SgdArg
 // in shared memory one user ahead by cp.async.  At the user's end a
 // reduce-scatter over the 4 groups leaves slice glane + 8 grp of the summed
 // user update on each lane, which writes L_i^c for that slice.
+//
+// Each warp takes one contiguous range of users, the ranges balanced by a
+// cost of entries plus kUserCost per user (found by a 16-way search of the
+// user offsets at the start), so that warps finish together whatever the
+// spread of entries per user.  The range is walked in units of kUnit users:
+// the metadata of the current unit sits in lanes [0, kUnit), that of the next
+// in lanes [kUnit, 2 kUnit), so the row staging and the entry window run on
+// across unit boundaries.
 #ifndef ESSPT_USERS4_MINB
 #define ESSPT_USERS4_MINB 3
 #endif
+constexpr int kUnit = 16;
+constexpr int32_t kUserCost = 5;
+
 __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdArgs a) {
   constexpr int NV = 4;
   __shared__ __align__(16) float4 stage[8][2][2][32];  // [warp][buffer][read row, base row][slice]
@@ -329,7 +340,6 @@ __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdA
   const int wib = threadIdx.x >> 5;
   const int glane = lane & 7;
   const int grp = lane >> 3;
-  const unsigned gmask = group_mask<8>(lane);
   const int32_t K4 = a.K >> 2;
   const int64_t slot4 = a.n_rows * K4;
   float4* ring4 = reinterpret_cast<float4*>(a.ring);
@@ -343,42 +353,89 @@ __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdA
   const bool my_act = my_q < K4;
   const uint64_t pol = policy_evict_first();
   float loss = 0.f;
-  const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
 
-  for (int64_t u0 = warp_id * 32; u0 < a.n_users; u0 += nwarps * 32) {
-    const int64_t uu = u0 + lane;
-    int32_t m_beg = 0, m_end = 0, m_vs = 0;
-    if (uu < a.n_users) {
-      m_beg = __ldg(a.uoff + uu);
-      m_end = __ldg(a.uoff + uu + 1);
-      m_vs = __ldg(a.v + __ldg(a.worker + uu)) % a.nslots;
+  // This warp's users [ua, ub): lanes 0..15 search the first user whose cost
+  // prefix uoff[u] + kUserCost u reaches the warp's share, lanes 16..31 the
+  // next warp's.  The cost prefix is strictly increasing, so the ranges tile
+  // [0, n_users).
+  int32_t ua, ub;
+  {
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int half = lane >> 4, hl = lane & 15;
+    const int64_t total = (int64_t)a.n_b + (int64_t)kUserCost * a.n_users;
+    const int64_t target = total * (w + half) / nw;
+    int32_t lo = 0, hi = a.n_users;  // answer in [lo, hi]; cost(hi) >= target
+    while (__any_sync(0xffffffffu, lo < hi)) {
+      const int32_t step = (hi - lo + 15) / 16;
+      const int32_t x = (int32_t)min((int64_t)lo + (int64_t)hl * step, (int64_t)hi);
+      const bool ge = lo < hi && (int64_t)__ldg(a.uoff + x) + (int64_t)kUserCost * x >= target;
+      const unsigned bits = (__ballot_sync(0xffffffffu, ge) >> (16 * half)) & 0xffffu;
+      if (lo < hi) {
+        if (bits == 0u) {
+          lo = (int32_t)min((int64_t)lo + (int64_t)15 * step, (int64_t)hi) + 1;
+        } else {
+          const int f = __ffs(bits) - 1;
+          const int32_t xf = (int32_t)min((int64_t)lo + (int64_t)f * step, (int64_t)hi);
+          if (f == 0) {
+            hi = lo;
+          } else {
+            lo = (int32_t)min((int64_t)lo + (int64_t)(f - 1) * step, (int64_t)hi) + 1;
+            hi = xf;
+          }
+        }
+      }
     }
-    const int32_t nusers = (int32_t)min((int64_t)32, (int64_t)a.n_users - u0);
-    Window<32> win;
+    ua = __shfl_sync(0xffffffffu, lo, 0);
+    ub = __shfl_sync(0xffffffffu, lo, 16);
+  }
+
+  // Entry range and read slot of users first.., into lanes [lo, lo + kUnit).
+  int32_t m_beg = 0, m_end = 0, m_vs = 0;
+  auto load_meta = [&](int64_t first, int lo) {
+    if (lane >= lo && lane < lo + kUnit) {
+      const int64_t uu = first + (lane - lo);
+      m_beg = m_end = m_vs = 0;
+      if (uu < ub) {
+        m_beg = __ldg(a.uoff + uu);
+        m_end = __ldg(a.uoff + uu + 1);
+        m_vs = __ldg(a.v + __ldg(a.worker + uu)) % a.nslots;
+      }
+    }
+  };
+  // Stage user u's rows (metadata in lane ml) into buffer b: lane l copies
+  // slice l of the read row (if it has entries) and of the base row (if it
+  // differs or is the only row needed).
+  auto stage_user = [&](int ml, int64_t u, int b) {
+    const int32_t vs = __shfl_sync(0xffffffffu, m_vs, ml);
+    const int32_t n = __shfl_sync(0xffffffffu, m_end, ml) - __shfl_sync(0xffffffffu, m_beg, ml);
+    const bool same = vs == a.slot_base && n > 0;
+    const bool in = lane < K4 && n <= kHeavy;
+    const float4* pv = ring4 + (int64_t)vs * slot4 + u * K4 + (lane < K4 ? lane : 0);
+    const float4* pb = base4 + u * K4 + (lane < K4 ? lane : 0);
+    cp_async16_hint(&stage[wib][b][0][lane], pv, in && n > 0, pol);
+    cp_async16_hint(&stage[wib][b][1][lane], pb, in && !same, pol);
+    cp_async_commit();
+  };
+
+  load_meta(ua, 0);
+  load_meta((int64_t)ua + kUnit, kUnit);
+  Window<32> win;
+  if (ua < ub) {
+    stage_user(0, ua, 0);
     win.reload(a, __shfl_sync(0xffffffffu, m_beg, 0), lane);
-
-    // Stage user t's rows into buffer b: lane l copies slice l of the read
-    // row (if it has entries) and of the base row (if it differs or is the
-    // only row needed).
-    auto stage_user = [&](int32_t t, int b) {
-      const int32_t vs = __shfl_sync(0xffffffffu, m_vs, t);
-      const int32_t n = __shfl_sync(0xffffffffu, m_end, t) - __shfl_sync(0xffffffffu, m_beg, t);
-      const bool same = vs == a.slot_base && n > 0;
-      const bool in = lane < K4 && n <= kHeavy;
-      const float4* pv = ring4 + (int64_t)vs * slot4 + (u0 + t) * K4 + (lane < K4 ? lane : 0);
-      const float4* pb = base4 + (u0 + t) * K4 + (lane < K4 ? lane : 0);
-      cp_async16_hint(&stage[wib][b][0][lane], pv, in && n > 0, pol);
-      cp_async16_hint(&stage[wib][b][1][lane], pb, in && !same, pol);
-      cp_async_commit();
-    };
-    stage_user(0, 0);
-
-    for (int32_t t = 0; t < nusers; ++t) {
-      const int b = t & 1;
+  }
+  int b = 0;
+  for (int64_t u0 = ua; u0 < ub; u0 += kUnit) {
+    const int32_t nusers = (int32_t)min((int64_t)kUnit, (int64_t)ub - u0);
+    for (int32_t t = 0; t < nusers; ++t, b ^= 1) {
       cp_async_wait_all();
       __syncwarp();
-      if (t + 1 < nusers) stage_user(t + 1, b ^ 1);
+      if (t + 1 < nusers) {
+        stage_user(t + 1, u0 + t + 1, b ^ 1);
+      } else if (u0 + kUnit < ub) {
+        stage_user(kUnit, u0 + kUnit, b ^ 1);
+      }
       const int32_t vs = __shfl_sync(0xffffffffu, m_vs, t);
       const int32_t beg = __shfl_sync(0xffffffffu, m_beg, t);
       const int32_t end = __shfl_sync(0xffffffffu, m_end, t);
@@ -445,6 +502,11 @@ __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdA
         st_stream_if(outq + (u0 + t) * K4 + my_q, f4_axpy(sc, g, lb), pol, my_act);
       }
     }
+    // The next unit's metadata moves down to lanes [0, kUnit).
+    m_beg = __shfl_down_sync(0xffffffffu, m_beg, kUnit);
+    m_end = __shfl_down_sync(0xffffffffu, m_end, kUnit);
+    m_vs = __shfl_down_sync(0xffffffffu, m_vs, kUnit);
+    load_meta(u0 + 2 * kUnit, kUnit);
     __syncwarp();
   }
   flush_loss(a.sq_loss, glane == 0 ? loss : 0.f, lane);
@@ -569,7 +631,14 @@ int grid_for(int64_t work_items, int64_t per_block, int max_per_sm) {
 template <int G, int NV>
 struct UsersF {
   static cudaError_t run4(const SgdArgs& a, cudaStream_t st) {
-    sgd_users4_kernel<<<grid_for(a.n_users, 256, 8), 256, 0, st>>>(a);
+    // One resident wave; the warps' user ranges are balanced in the kernel.
+    static int per_sm = 0;
+    if (per_sm == 0) {
+      if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sgd_users4_kernel, 256, 0) != cudaSuccess ||
+          per_sm <= 0)
+        per_sm = 1;
+    }
+    sgd_users4_kernel<<<grid_for((a.n_users + kUnit - 1) / kUnit, 8, per_sm), 256, 0, st>>>(a);
     return cudaGetLastError();
   }
   static cudaError_t run(const SgdArgs& a, cudaStream_t st) {
