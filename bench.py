@@ -314,7 +314,7 @@ def run_gpu(args, w):
     floor_avg = statistics.mean(floors)
     peak, peak_kind = _peaks()
     achieved = floor_avg / kern_avg_s / 1e9
-    kernel = "sgd_users4_kernel" if 64 < w.K <= 128 else "sgd_users_kernel"
+    kernel = "sgd_users32_kernel" if 64 < w.K <= 128 else "sgd_users_kernel"
     n_avg = ratings / K
     B_model = 12 + 16 * w.K + 8 * w.K * (w.n_users + w.n_items) / n_avg
     out = {

@@ -1,7 +1,8 @@
 // Matrix-factorisation SGD on the version ring (Sec. 3.1 updates under the
 // SSP / ESSP read schedule).  One clock is:
 //   sgd_chunks_kernel   entries of very active users, in chunks (if any);
-//   sgd_users_kernel    every other user: its row of version c, written once;
+//   sgd_users_kernel    every other user: its row of version c, written once
+//                       (sgd_users32_kernel for rows of 68..128 values);
 //   heavy_merge_kernel  rows of the very active users (if any);
 //   item_merge_kernel   the Clock() merge of the item rows.
 // Item-row (and heavy-user) deltas are summed, unscaled, into zero-initialised
@@ -312,13 +313,19 @@ __global__ void __launch_bounds__(256, ESSPT_USERS_MINB) sgd_users_kernel(SgdArg
   flush_loss(a.sq_loss, glane == 0 ? loss : 0.f, lane);
 }
 
-// Rows of 68..128 values (17..32 float4 slices): a group of 8 lanes holds
-// one row, 4 slices per lane (slice q = glane + 8k), and the warp's 4 groups
-// take 4 entries of the same user per step, so one 3-level reduction serves
-// 4 dot products.  The user's rows at the read and base versions are staged
-// in shared memory one user ahead by cp.async.  At the user's end a
-// reduce-scatter over the 4 groups leaves slice glane + 8 grp of the summed
-// user update on each lane, which writes L_i^c for that slice.
+#ifndef ESSPT_USERS32_MINB
+#define ESSPT_USERS32_MINB 3
+#endif
+constexpr int kUnit = 16;
+constexpr int32_t kUserCost = 5;
+
+// Rows of 68..128 values (17..32 float4 slices), one slice per lane: the
+// whole warp holds one user's row (lane l owns slice l of L_i and of its
+// update sum) and takes 4 of the user's entries per step, gathering each item
+// row with one coalesced load.  The 4 partial dot products are reduced with
+// a transposing butterfly (6 shuffles) that leaves entry q's dot product on
+// lanes 8q .. 8q+7.  The user's rows at the read and base versions are staged
+// in shared memory one user ahead by cp.async.
 //
 // Each warp takes one contiguous range of users, the ranges balanced by a
 // cost of entries plus kUserCost per user (found by a 16-way search of the
@@ -327,37 +334,21 @@ __global__ void __launch_bounds__(256, ESSPT_USERS_MINB) sgd_users_kernel(SgdArg
 // the metadata of the current unit sits in lanes [0, kUnit), that of the next
 // in lanes [kUnit, 2 kUnit), so the row staging and the entry window run on
 // across unit boundaries.
-#ifndef ESSPT_USERS4_MINB
-#define ESSPT_USERS4_MINB 3
-#endif
-constexpr int kUnit = 16;
-constexpr int32_t kUserCost = 5;
-
-__global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdArgs a) {
-  constexpr int NV = 4;
+__global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(SgdArgs a) {
   __shared__ __align__(16) float4 stage[8][2][2][32];  // [warp][buffer][read row, base row][slice]
   const int lane = threadIdx.x & 31;
   const int wib = threadIdx.x >> 5;
-  const int glane = lane & 7;
-  const int grp = lane >> 3;
+  const int q = lane >> 3;  // the entry of a step whose dot product this lane ends up with
   const int32_t K4 = a.K >> 2;
+  const bool on = lane < K4;
   const int64_t slot4 = a.n_rows * K4;
   float4* ring4 = reinterpret_cast<float4*>(a.ring);
   float4* outq = ring4 + (int64_t)a.slot_out * slot4;
   const float4* base4 = ring4 + (int64_t)a.slot_base * slot4;
-  float4* dRq = reinterpret_cast<float4*>(a.dR) + glane;
-  bool act[NV];
-#pragma unroll
-  for (int k = 0; k < NV; ++k) act[k] = glane + 8 * k < K4;
-  const int my_q = glane + 8 * grp;  // the slice this lane writes
-  const bool my_act = my_q < K4;
+  float4* dRq = reinterpret_cast<float4*>(a.dR) + lane;
   const uint64_t pol = policy_evict_first();
   float loss = 0.f;
 
-  // This warp's users [ua, ub): lanes 0..15 search the first user whose cost
-  // prefix uoff[u] + kUserCost u reaches the warp's share, lanes 16..31 the
-  // next warp's.  The cost prefix is strictly increasing, so the ranges tile
-  // [0, n_users).
   int32_t ua, ub;
   {
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -365,7 +356,7 @@ __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdA
     const int half = lane >> 4, hl = lane & 15;
     const int64_t total = (int64_t)a.n_b + (int64_t)kUserCost * a.n_users;
     const int64_t target = total * (w + half) / nw;
-    int32_t lo = 0, hi = a.n_users;  // answer in [lo, hi]; cost(hi) >= target
+    int32_t lo = 0, hi = a.n_users;
     while (__any_sync(0xffffffffu, lo < hi)) {
       const int32_t step = (hi - lo + 15) / 16;
       const int32_t x = (int32_t)min((int64_t)lo + (int64_t)hl * step, (int64_t)hi);
@@ -390,7 +381,6 @@ __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdA
     ub = __shfl_sync(0xffffffffu, lo, 16);
   }
 
-  // Entry range and read slot of users first.., into lanes [lo, lo + kUnit).
   int32_t m_beg = 0, m_end = 0, m_vs = 0;
   auto load_meta = [&](int64_t first, int lo) {
     if (lane >= lo && lane < lo + kUnit) {
@@ -403,16 +393,13 @@ __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdA
       }
     }
   };
-  // Stage user u's rows (metadata in lane ml) into buffer b: lane l copies
-  // slice l of the read row (if it has entries) and of the base row (if it
-  // differs or is the only row needed).
   auto stage_user = [&](int ml, int64_t u, int b) {
     const int32_t vs = __shfl_sync(0xffffffffu, m_vs, ml);
     const int32_t n = __shfl_sync(0xffffffffu, m_end, ml) - __shfl_sync(0xffffffffu, m_beg, ml);
     const bool same = vs == a.slot_base && n > 0;
-    const bool in = lane < K4 && n <= kHeavy;
-    const float4* pv = ring4 + (int64_t)vs * slot4 + u * K4 + (lane < K4 ? lane : 0);
-    const float4* pb = base4 + u * K4 + (lane < K4 ? lane : 0);
+    const bool in = on && n <= kHeavy;
+    const float4* pv = ring4 + (int64_t)vs * slot4 + u * K4 + (on ? lane : 0);
+    const float4* pb = base4 + u * K4 + (on ? lane : 0);
     cp_async16_hint(&stage[wib][b][0][lane], pv, in && n > 0, pol);
     cp_async16_hint(&stage[wib][b][1][lane], pb, in && !same, pol);
     cp_async_commit();
@@ -441,75 +428,67 @@ __global__ void __launch_bounds__(256, ESSPT_USERS4_MINB) sgd_users4_kernel(SgdA
       const int32_t end = __shfl_sync(0xffffffffu, m_end, t);
       const int32_t n = end - beg;
       if (n > kHeavy) continue;
-      const float4* Lv_s = &stage[wib][b][0][glane];
-      const float4* Rq = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4 + glane;
-      float4 gL[NV];
-#pragma unroll
-      for (int k = 0; k < NV; ++k) gL[k] = f4_zero();
+      const float4 Lv = stage[wib][b][0][lane];
+      const float4* Rq = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4 + lane;
+      float4 gL = f4_zero();
       for (int32_t tt = beg; tt < end;) {
         win.cover(a, tt, lane);
         const int32_t cnt = min(4, min(end - tt, win.W + 32 - tt));
-        const bool valid = grp < cnt;
-        const int src = min(tt - win.W + grp, 31);
-        const int32_t j = __shfl_sync(0xffffffffu, win.cj, src);
-        const float d = __shfl_sync(0xffffffffu, win.cd, src);
-        const int32_t dst = __shfl_sync(0xffffffffu, win.cdst, src);
-        const float4* row = Rq + j * K4;
-        float4 R[NV];
+        const int w0 = tt - win.W;
+        float4 R[4];
+        int32_t dst[4];
+        float p[4];
 #pragma unroll
-        for (int k = 0; k < NV; ++k) R[k] = (act[k] && valid) ? __ldg(row + 8 * k) : f4_zero();
-        float part = 0.f;
+        for (int e4 = 0; e4 < 4; ++e4) {
+          const int src = min(w0 + e4, 31);
+          const int32_t j = __shfl_sync(0xffffffffu, win.cj, src);
+          dst[e4] = __shfl_sync(0xffffffffu, win.cdst, src);
+          R[e4] = (on && e4 < cnt) ? __ldg(Rq + j * K4) : f4_zero();
+          p[e4] = dot4(Lv, R[e4]);
+        }
+        // Transposing butterfly: lanes with bit 4 clear keep entries {0, 1},
+        // the others {2, 3}; then bit 3 picks one of the pair; the last three
+        // levels sum over the 8 lanes that share bits 3 and 4.
+        const bool h4 = lane & 16, h3 = lane & 8;
+        float k0 = h4 ? p[2] : p[0], k1 = h4 ? p[3] : p[1];
+        k0 += __shfl_xor_sync(0xffffffffu, h4 ? p[0] : p[2], 16);
+        k1 += __shfl_xor_sync(0xffffffffu, h4 ? p[1] : p[3], 16);
+        float dot = h3 ? k1 : k0;
+        dot += __shfl_xor_sync(0xffffffffu, h3 ? k0 : k1, 8);
+        dot += __shfl_xor_sync(0xffffffffu, dot, 4);
+        dot += __shfl_xor_sync(0xffffffffu, dot, 2);
+        dot += __shfl_xor_sync(0xffffffffu, dot, 1);
+        const float dq = __shfl_sync(0xffffffffu, win.cd, min(w0 + q, 31));
+        const float eq = q < cnt ? dq - dot : 0.f;
+        if ((lane & 7) == 0) loss += eq * eq;
 #pragma unroll
-        for (int k = 0; k < NV; ++k) part += dot4(Lv_s[8 * k], R[k]);
-#pragma unroll
-        for (int off = 4; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
-        const float e = valid ? d - part : 0.f;
-        loss += e * e;
-        float4* out = dRq + dst * a.dR_ld;
-#pragma unroll
-        for (int k = 0; k < NV; ++k) {
-          const float4 r = R[k], l = Lv_s[8 * k];
-          gL[k].x += e * r.x;
-          gL[k].y += e * r.y;
-          gL[k].z += e * r.z;
-          gL[k].w += e * r.w;
-          red_add_v4_if(out + 8 * k,
-                        make_float4(e * l.x - a.lambda * r.x, e * l.y - a.lambda * r.y, e * l.z - a.lambda * r.z,
-                                    e * l.w - a.lambda * r.w),
-                        act[k] && valid);
+        for (int e4 = 0; e4 < 4; ++e4) {
+          const float e = __shfl_sync(0xffffffffu, eq, 8 * e4);
+          const float4 r = R[e4];
+          gL.x += e * r.x;
+          gL.y += e * r.y;
+          gL.z += e * r.z;
+          gL.w += e * r.w;
+          red_add_v4_if(dRq + dst[e4] * a.dR_ld,
+                        make_float4(e * Lv.x - a.lambda * r.x, e * Lv.y - a.lambda * r.y,
+                                    e * Lv.z - a.lambda * r.z, e * Lv.w - a.lambda * r.w),
+                        on && e4 < cnt);
         }
         tt += cnt;
       }
-      // Reduce-scatter over the groups: group g keeps slice set k = g.
-      {
-        const bool hi = grp >= 2;
-        float4 k0 = hi ? gL[2] : gL[0], k1 = hi ? gL[3] : gL[1];
-        const float4 s0 = hi ? gL[0] : gL[2], s1 = hi ? gL[1] : gL[3];
-        k0 = f4_add(k0, make_float4(__shfl_xor_sync(0xffffffffu, s0.x, 16), __shfl_xor_sync(0xffffffffu, s0.y, 16),
-                                    __shfl_xor_sync(0xffffffffu, s0.z, 16), __shfl_xor_sync(0xffffffffu, s0.w, 16)));
-        k1 = f4_add(k1, make_float4(__shfl_xor_sync(0xffffffffu, s1.x, 16), __shfl_xor_sync(0xffffffffu, s1.y, 16),
-                                    __shfl_xor_sync(0xffffffffu, s1.z, 16), __shfl_xor_sync(0xffffffffu, s1.w, 16)));
-        const bool odd = grp & 1;
-        float4 keep = odd ? k1 : k0;
-        const float4 snd = odd ? k0 : k1;
-        keep = f4_add(keep, make_float4(__shfl_xor_sync(0xffffffffu, snd.x, 8), __shfl_xor_sync(0xffffffffu, snd.y, 8),
-                                        __shfl_xor_sync(0xffffffffu, snd.z, 8), __shfl_xor_sync(0xffffffffu, snd.w, 8)));
-        const bool same = vs == a.slot_base && n > 0;
-        const float4 lv = stage[wib][b][0][my_q];
-        const float4 lb = stage[wib][b][same ? 0 : 1][my_q];
-        const float sc = a.eta * cap_scale(a.cap, n);
-        const float4 g = f4_axpy(-(float)n * a.lambda, lv, keep);
-        st_stream_if(outq + (u0 + t) * K4 + my_q, f4_axpy(sc, g, lb), pol, my_act);
-      }
+      const bool same = vs == a.slot_base && n > 0;
+      const float4 lb = stage[wib][b][same ? 0 : 1][lane];
+      const float sc = a.eta * cap_scale(a.cap, n);
+      const float4 g = f4_axpy(-(float)n * a.lambda, Lv, gL);
+      st_stream_if(outq + (u0 + t) * K4 + lane, f4_axpy(sc, g, lb), pol, on);
     }
-    // The next unit's metadata moves down to lanes [0, kUnit).
     m_beg = __shfl_down_sync(0xffffffffu, m_beg, kUnit);
     m_end = __shfl_down_sync(0xffffffffu, m_end, kUnit);
     m_vs = __shfl_down_sync(0xffffffffu, m_vs, kUnit);
     load_meta(u0 + 2 * kUnit, kUnit);
     __syncwarp();
   }
-  flush_loss(a.sq_loss, glane == 0 ? loss : 0.f, lane);
+  flush_loss(a.sq_loss, loss, lane);
 }
 
 // Chunks of at most kChunk entries of users with more than kHeavy entries:
@@ -628,19 +607,21 @@ int grid_for(int64_t work_items, int64_t per_block, int max_per_sm) {
   return (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sm_count() * max_per_sm));
 }
 
+// One resident wave of sgd_users32_kernel; its warps balance the users among
+// themselves.
+cudaError_t run_users32(const SgdArgs& a, cudaStream_t st) {
+  static int per_sm = 0;
+  if (per_sm == 0) {
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sgd_users32_kernel, 256, 0) != cudaSuccess ||
+        per_sm <= 0)
+      per_sm = 1;
+  }
+  sgd_users32_kernel<<<grid_for((a.n_users + kUnit - 1) / kUnit, 8, per_sm), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
 template <int G, int NV>
 struct UsersF {
-  static cudaError_t run4(const SgdArgs& a, cudaStream_t st) {
-    // One resident wave; the warps' user ranges are balanced in the kernel.
-    static int per_sm = 0;
-    if (per_sm == 0) {
-      if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sgd_users4_kernel, 256, 0) != cudaSuccess ||
-          per_sm <= 0)
-        per_sm = 1;
-    }
-    sgd_users4_kernel<<<grid_for((a.n_users + kUnit - 1) / kUnit, 8, per_sm), 256, 0, st>>>(a);
-    return cudaGetLastError();
-  }
   static cudaError_t run(const SgdArgs& a, cudaStream_t st) {
     // 8 warps per block, 32 users per warp
     sgd_users_kernel<G, NV><<<grid_for(a.n_users, 256, 8), 256, 0, st>>>(a);
@@ -666,13 +647,7 @@ cudaError_t dispatch_k(int32_t K, const Arg& a, cudaStream_t st) {
   if (K4 <= 4) return F<4, 1>::run(a, st);
   if (K4 <= 8) return F<8, 1>::run(a, st);
   if (K4 <= 16) return F<16, 1>::run(a, st);
-#if defined(ESSPT_WIDE_ROWS)
-  if (K4 <= 32) return F<16, 2>::run(a, st);
-#elif defined(ESSPT_QUAD_ROWS)
-  if (K4 <= 32) return F<8, 4>::run(a, st);
-#else
   if (K4 <= 32) return F<32, 1>::run(a, st);
-#endif
   if (K4 <= 64) return F<32, 2>::run(a, st);
   if (K4 <= 96) return F<32, 3>::run(a, st);
   return F<32, 4>::run(a, st);
@@ -681,9 +656,7 @@ cudaError_t dispatch_k(int32_t K, const Arg& a, cudaStream_t st) {
 }  // namespace
 
 cudaError_t launch_sgd_users(const SgdArgs& a, cudaStream_t st) {
-#ifndef ESSPT_NO_USERS4
-  if (a.K > 64 && a.K <= 128) return UsersF<8, 4>::run4(a, st);
-#endif
+  if (a.K > 64 && a.K <= 128) return run_users32(a, st);
   return dispatch_k<UsersF>(a.K, a, st);
 }
 cudaError_t launch_sgd_chunks(const ChunkArgs& c, cudaStream_t st) { return dispatch_k<ChunksF>(c.a.K, c, st); }

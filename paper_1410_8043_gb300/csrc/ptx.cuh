@@ -65,11 +65,12 @@ __device__ __forceinline__ void st_stream_if(float4* p, float4 v, uint64_t pol, 
       : "memory");
 }
 
-// out[0..3] += v when `pred`, performed at L2.  The return value of the
-// vector atomicAdd (sm_90 and later) is unused, so it issues as a reduction;
-// the compiler predicates it without a branch.
+// out[0..3] += v when `pred`, performed at L2 (vector reduction, sm_90 and
+// later), predicated inside the asm so that no branch surrounds it.
 __device__ __forceinline__ void red_add_v4_if(float4* p, float4 v, bool pred) {
-  if (pred) atomicAdd(p, v);
+  asm volatile("{\n .reg .pred q;\n setp.ne.b32 q, %5, 0;\n @q red.global.add.v4.f32 [%0], {%1,%2,%3,%4};\n}" ::"l"(p),
+               "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"((int)pred)
+               : "memory");
 }
 
 // 16-byte asynchronous global -> shared copy (bypassing L1); when `pred` is
