@@ -10,6 +10,7 @@
 // L2 addresses; the merges apply eta, the hot-row scale and the sum of the
 // replicas, then clear them for the next clock.
 #include <algorithm>
+#include <type_traits>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -48,6 +49,10 @@ __device__ __forceinline__ float4 f4_axpy(float s, float4 x, float4 y) {  // y +
 __device__ __forceinline__ float cap_scale(int32_t cap, int32_t n) {
   return (cap > 0 && n > cap) ? (float)cap / (float)n : 1.f;
 }
+
+// cap / n for a row past the cap, out of line: the rare case stays off the
+// common path.
+__device__ __noinline__ float capped_scale(int32_t cap, int32_t n) { return (float)cap / (float)n; }
 
 // Entry t of the minibatch: item, value and the replica row its item update
 // adds into; zeros past the end.
@@ -429,21 +434,26 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
       const int32_t n = end - beg;
       if (n > kHeavy) continue;
       const float4 Lv = stage[wib][b][0][lane];
-      const float4* Rq = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4 + lane;
+      // Lanes past the row end read slice 0 (their staged L is zero), so the
+      // item-row loads need no predicate.
+      const float4* Rq = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4 + (on ? lane : 0);
       float4 gL = f4_zero();
-      for (int32_t tt = beg; tt < end;) {
-        win.cover(a, tt, lane);
-        const int32_t cnt = min(4, min(end - tt, win.W + 32 - tt));
+      // One step: entries tt .. tt+cnt-1 of the user.  It is compiled twice,
+      // for full steps (cnt = 4, the common case) and for the user's last,
+      // partial one, whose missing entries read a row of the window (any
+      // valid one), get e = 0 and add nothing.
+      auto step = [&](auto full_tag, int32_t tt, int32_t cnt) {
+        constexpr bool kFull = decltype(full_tag)::value;
         const int w0 = tt - win.W;
         float4 R[4];
         int32_t dst[4];
         float p[4];
 #pragma unroll
         for (int e4 = 0; e4 < 4; ++e4) {
-          const int src = min(w0 + e4, 31);
+          const int src = kFull ? w0 + e4 : min(w0 + e4, 31);
           const int32_t j = __shfl_sync(0xffffffffu, win.cj, src);
           dst[e4] = __shfl_sync(0xffffffffu, win.cdst, src);
-          R[e4] = (on && e4 < cnt) ? __ldg(Rq + j * K4) : f4_zero();
+          R[e4] = __ldg(Rq + j * K4);
           p[e4] = dot4(Lv, R[e4]);
         }
         // Transposing butterfly: lanes with bit 4 clear keep entries {0, 1},
@@ -458,8 +468,8 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
         dot += __shfl_xor_sync(0xffffffffu, dot, 4);
         dot += __shfl_xor_sync(0xffffffffu, dot, 2);
         dot += __shfl_xor_sync(0xffffffffu, dot, 1);
-        const float dq = __shfl_sync(0xffffffffu, win.cd, min(w0 + q, 31));
-        const float eq = q < cnt ? dq - dot : 0.f;
+        const float dq = __shfl_sync(0xffffffffu, win.cd, kFull ? w0 + q : min(w0 + q, 31));
+        const float eq = (kFull || q < cnt) ? dq - dot : 0.f;
         if ((lane & 7) == 0) loss += eq * eq;
 #pragma unroll
         for (int e4 = 0; e4 < 4; ++e4) {
@@ -472,13 +482,23 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
           red_add_v4_if(dRq + dst[e4] * a.dR_ld,
                         make_float4(e * Lv.x - a.lambda * r.x, e * Lv.y - a.lambda * r.y,
                                     e * Lv.z - a.lambda * r.z, e * Lv.w - a.lambda * r.w),
-                        on && e4 < cnt);
+                        on && (kFull || e4 < cnt));
+        }
+      };
+      for (int32_t tt = beg; tt < end;) {
+        win.cover(a, tt, lane);
+        const int32_t cnt = min(4, min(end - tt, win.W + 32 - tt));
+        if (cnt == 4) {
+          step(std::true_type{}, tt, cnt);
+        } else {
+          step(std::false_type{}, tt, cnt);
         }
         tt += cnt;
       }
       const bool same = vs == a.slot_base && n > 0;
       const float4 lb = stage[wib][b][same ? 0 : 1][lane];
-      const float sc = a.eta * cap_scale(a.cap, n);
+      float sc = a.eta;
+      if (a.cap > 0 && n > a.cap) sc = a.eta * capped_scale(a.cap, n);
       const float4 g = f4_axpy(-(float)n * a.lambda, Lv, gL);
       st_stream_if(outq + (u0 + t) * K4 + lane, f4_axpy(sc, g, lb), pol, on);
     }
@@ -609,9 +629,17 @@ int grid_for(int64_t work_items, int64_t per_block, int max_per_sm) {
 
 // One resident wave of sgd_users32_kernel; its warps balance the users among
 // themselves.
+#ifndef ESSPT_U32_CARVEOUT
+#define ESSPT_U32_CARVEOUT 25
+#endif
 cudaError_t run_users32(const SgdArgs& a, cudaStream_t st) {
   static int per_sm = 0;
   if (per_sm == 0) {
+    // Ask for the smallest shared-memory carveout that holds the resident
+    // blocks' staging buffers (percent of the maximum), leaving the rest of
+    // the SM's memory to L1, which caches the gathered item rows.
+    if (ESSPT_U32_CARVEOUT >= 0)
+      cudaFuncSetAttribute(sgd_users32_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, ESSPT_U32_CARVEOUT);
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sgd_users32_kernel, 256, 0) != cudaSuccess ||
         per_sm <= 0)
       per_sm = 1;
