@@ -31,10 +31,10 @@ METRIC = "SGD ratings/sec per clock on 1 GB300; achieved HBM GB/s vs peak"
 UNIT = "ratings/s"
 
 
-def _profiled_traffic(kernel: str):
-    """DRAM bytes per launch of `kernel` from its committed ncu summary under
-    profiles/, or None when the kernel source changed since the capture."""
-    import glob
+def _profiled_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch of `kernel` on `workload` from its committed ncu
+    summary profiles/<kernel>_<workload>.md, or None when there is none or the
+    kernel source changed since the capture."""
     import hashlib
 
     src = os.path.join(ROOT, "paper_1410_8043_gb300", "csrc", "mf_kernels.cu")
@@ -42,7 +42,9 @@ def _profiled_traffic(kernel: str):
         digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
     except OSError:
         return None
-    for path in glob.glob(os.path.join(ROOT, "profiles", f"{kernel}_*.md")):
+    for path in [os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")]:
+        if not os.path.exists(path):
+            continue
         fields = {}
         for line in open(path):
             if ":" in line and not line.startswith(("|", "#", " ", "`")):
@@ -202,6 +204,14 @@ class FloorModel:
         return 12 * int(self.n[b]) + 8 * w.K * w.n_users + 4 * w.K * (users + items), int(self.n[b])
 
 
+def _vap_launches(w, c):
+    """Kernels VAP adds to clock c: the norms for clock c+1 and its schedule."""
+    if w.model != "vap":
+        return 0
+    kmax = min(w.s, c)
+    return (kmax + 7) // 8 + 1
+
+
 def run_gpu(args, w):
     import torch
 
@@ -332,7 +342,9 @@ def run_gpu(args, w):
         "data": "synthetic (seeded counter generator; Netflix-shaped, no real records)",
         "config": {
             "workload": f"{w.name}: {w.n_users}x{w.n_items}, {w.n_obs} entries, rank {w.K}, P={w.P}, "
-                        f"F={w.F}, {w.model.upper()} s={w.s}, eta={w.eta}, lambda={w.lam}, cap={w.cap}",
+                        f"F={w.F}, {w.model.upper()} s={w.s}"
+                        + (f" v0={w.vap_v0}" if w.model == "vap" else "")
+                        + f", eta={w.eta}, lambda={w.lam}, cap={w.cap}",
             "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
             "l2": "inputs larger than L2 (version ring %.2f GB, entries %.2f GB; ~%.0f MB streamed per clock)"
                   % ((w.s + 2) * (w.n_users + w.n_items) * w.K * 4 / 1e9, w.n_obs * 12 / 1e9, floor_avg / 1e6),
@@ -346,7 +358,7 @@ def run_gpu(args, w):
             "peak_kind": peak_kind,
             "unit": "GB/s",
             "frac": achieved / peak,
-            "traffic": _profiled_traffic(kernel),
+            "traffic": _profiled_traffic(kernel, w.name),
             "algorithmic_bytes_per_launch": floor_avg,
             "kernel_ms": statistics.mean(kern_ms),
             "modelled_bytes_per_rating": B_model,
@@ -355,8 +367,10 @@ def run_gpu(args, w):
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d // K, "d2h_bytes_per_step": d2h // K},
         # per clock: the SGD kernel and the item merge (which also computes the
         # next schedule), plus the chunk and heavy-merge kernels on minibatches
-        # with heavy users
-        "gpu_launches": int(sum(2 + 2 * model.heavy[(c - 1) % w.F] for c in range(W + 1, W + K + 1))),
+        # with heavy users; VAP adds its norm kernel (one per 8 candidate
+        # versions) and the schedule kernel after the merge
+        "gpu_launches": int(sum(2 + 2 * model.heavy[(c - 1) % w.F] + _vap_launches(w, c)
+                                for c in range(W + 1, W + K + 1))),
         "clocks": clocks,
         "objective": {"clock": c_final, "sq_loss": sq, "penalised": pen},
         # Fig. 1 (left) quantity: clock differential v_p(c) - c of every read in

@@ -7,6 +7,7 @@
          1/20 per clock, SSP s=3, 40 clocks.
 * mid_essp: the mid data under ESSP (eager push), Geometric(0.7) delays
          clamped to [0, 3].
+* mid_vap: the mid data under the VAP value bound 0.3 / sqrt(c), s=3.
 * large: 10M x 1M, 2B entries, Zipf(1.1) users and items, rank-64 model,
          128 workers, 1/50 per clock, SSP s=4, 20 clocks.
 * sweep: the mid data with s in {0,1,2,4,8} x P in {1,8,64,512} x {SSP, ESSP},
@@ -33,7 +34,7 @@ class Workload:
     P: int
     F: int
     s: int
-    model: str  # "ssp" (lazy pull) or "essp" (eager push)
+    model: str  # "ssp" (lazy pull), "essp" (eager push) or "vap" (value bound)
     clocks: int
     eta: float
     lam: float
@@ -48,6 +49,7 @@ class Workload:
     sched_seed: int = SCHED_SEED
     essp_p: float = 0.7
     essp_max_delay: int = 3
+    vap_v0: float = 0.0  # "vap": initial value bound v0 (bound v0 / sqrt(c) at clock c)
 
     def with_(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
@@ -97,6 +99,12 @@ WORKLOADS = {
     "mid_essp": Workload(
         "mid_essp", 480_000, 18_000, 100_000_000, K=100, P=32, F=20, s=3, model="essp",
         clocks=40, eta=0.005, lam=0.05, cap=20, data=_MID_DATA,
+    ),
+    # VAP read schedule (Sec. 2.1) on the mid data: v0 = 0.3 gives reads of
+    # staleness 0..3 over the first clocks, then a mix of 2 and 3.
+    "mid_vap": Workload(
+        "mid_vap", 480_000, 18_000, 100_000_000, K=100, P=32, F=20, s=3, model="vap",
+        clocks=40, eta=0.005, lam=0.05, cap=20, data=_MID_DATA, vap_v0=0.3,
     ),
     "large": Workload(
         "large", 10_000_000, 1_000_000, 2_000_000_000, K=64, P=128, F=50, s=4,

@@ -59,6 +59,15 @@ typedef enum {
   ESSPT_ESSP_EAGER = 1,
   /* The caller supplies every v_p(c) with esspt_set_schedule(). */
   ESSPT_EXTERNAL = 2,
+  /* VAP, the value-bounded model (Sec. 2.1): a worker that reads version v
+   * at clock c has the updates X[c-1] - X[v] in transit.  Every worker reads
+   * the stalest v in [max(0, c-1-s), c-1] whose in-transit max-norm
+   * |X[c-1] - X[v]|_inf (over the whole table, fp32) is at most
+   * vap_v0 / sqrt(c), the shrinking bound v_t = v0 / sqrt(t) of the
+   * SGD-under-VAP theorem (Sec. 3).  Version c-1 always qualifies; a NaN
+   * norm never does.  Each clock reads the s+1 candidate versions once more
+   * to compute the norms (the cost the paper names for VAP). */
+  ESSPT_VAP = 3,
 } esspt_model;
 
 typedef struct {
@@ -72,6 +81,7 @@ typedef struct {
   double essp_p;          /* ESSPT_ESSP_EAGER: success probability in (0, 1] */
   uint64_t seed;          /* seed of the schedule's counter generator (SplitMix64) */
   void* stream;           /* cudaStream_t; NULL = legacy default stream */
+  double vap_v0;          /* ESSPT_VAP: initial value bound v0 >= 0 */
 } esspt_config;
 
 typedef struct esspt_ctx esspt_ctx;

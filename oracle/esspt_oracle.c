@@ -14,7 +14,13 @@
  *     after a delay of delta_{p,c} ~ Geometric(p) clocks clamped to
  *     [0, min(max_delay, s)]; the read version never goes backwards;
  *   - all entries of a worker in one clock read the same version and both
- *     updates use the old L_i and R_j (no read-my-writes, Sec. 3 footnote).
+ *     updates use the old L_i and R_j (no read-my-writes, Sec. 3 footnote);
+ *   - VAP (Sec. 2.1): a worker reading version v at clock c has the updates
+ *     X[c-1] - X[v] in transit; in this lockstep simulation every worker
+ *     refreshes as lazily as the value bound allows, i.e. reads the stalest
+ *     version inside the staleness window whose in-transit max-norm is at
+ *     most v0 / sqrt(c) (the shrinking bound v_t = v0 / sqrt(t) of the
+ *     SGD-under-VAP theorem, Sec. 3, with t = c); a NaN norm never qualifies.
  */
 #include "esspt_oracle.h"
 
@@ -58,6 +64,8 @@ struct orc_state {
   int32_t* v_prev;  /* read versions of the last clock (P) */
   double* delta;    /* rows * K */
   int64_t* count;   /* rows, entries per row in this clock */
+  double* vap_norm; /* s+1, ORC_VAP norms of the last clock */
+  double vap_bound; /* ORC_VAP bound of the last clock */
 };
 
 static double* orc_slot(const orc_state* st, int32_t version) {
@@ -108,11 +116,52 @@ int orc_schedule_rule(const orc_config* cfg, int32_t c, const int32_t* v_prev, i
   return 0;
 }
 
+/* ORC_VAP read version of clock c: the stalest v in the window whose
+ * in-transit max-norm |X[c-1] - X[v]|_inf is at most v0 / sqrt(c). */
+static int32_t orc_vap_version(orc_state* st, int32_t c) {
+  const orc_config* cfg = &st->cfg;
+  const int64_t n = st->rows * cfg->K;
+  const double* cur = orc_slot(st, c - 1);
+  const double bound = cfg->vap_v0 / sqrt((double)c);
+  int32_t v = c - 1;
+  for (int32_t k = 0; k <= cfg->s; ++k) st->vap_norm[k] = 0.0;
+  st->vap_bound = bound;
+  for (int32_t k = cfg->s; k >= 1; --k) {
+    if (c - 1 - k < 0) continue;
+    const double* old = orc_slot(st, c - 1 - k);
+    double m = 0.0;
+    for (int64_t x = 0; x < n; ++x) {
+      double d = fabs(cur[x] - old[x]);
+      if (d != d) {
+        m = d;
+        break;
+      }
+      if (d > m) m = d;
+    }
+    st->vap_norm[k] = m;
+  }
+  for (int32_t k = cfg->s; k >= 1; --k) {
+    if (c - 1 - k < 0) continue;
+    if (st->vap_norm[k] <= bound) {
+      v = c - 1 - k;
+      break;
+    }
+  }
+  return v;
+}
+
+int orc_vap_norms(const orc_state* st, double* out, double* bound) {
+  if (st->cfg.model != ORC_VAP || st->version < 1) return -1;
+  memcpy(out, st->vap_norm, (size_t)(st->cfg.s + 1) * sizeof(double));
+  *bound = st->vap_bound;
+  return 0;
+}
+
 orc_state* orc_create(const orc_config* cfg, int64_t n_obs, const int32_t* i, const int32_t* j,
                       const float* D, const uint8_t* minibatch, const int32_t* user_worker,
                       const float* L0, const float* R0) {
   if (!cfg || cfg->n_users <= 0 || cfg->n_items <= 0 || cfg->K <= 0 || cfg->P <= 0 || cfg->s < 0 ||
-      cfg->F <= 0 || n_obs < 0 || cfg->model < 0 || cfg->model > ORC_EXTERNAL)
+      cfg->F <= 0 || n_obs < 0 || cfg->model < 0 || cfg->model > ORC_VAP || (cfg->model == ORC_VAP && !(cfg->vap_v0 >= 0.0)))
     return NULL;
   orc_state* st = (orc_state*)calloc(1, sizeof(orc_state));
   if (!st) return NULL;
@@ -131,7 +180,8 @@ orc_state* orc_create(const orc_config* cfg, int64_t n_obs, const int32_t* i, co
   st->v_prev = (int32_t*)calloc((size_t)cfg->P, sizeof(int32_t));
   st->delta = (double*)calloc((size_t)(st->rows * K), sizeof(double));
   st->count = (int64_t*)calloc((size_t)st->rows, sizeof(int64_t));
-  if (!st->tables || !st->v_prev || !st->delta || !st->count) {
+  st->vap_norm = (double*)calloc((size_t)cfg->s + 1, sizeof(double));
+  if (!st->tables || !st->v_prev || !st->delta || !st->count || !st->vap_norm) {
     orc_destroy(st);
     return NULL;
   }
@@ -150,6 +200,7 @@ void orc_destroy(orc_state* st) {
   free(st->v_prev);
   free(st->delta);
   free(st->count);
+  free(st->vap_norm);
   free(st);
 }
 
@@ -180,6 +231,9 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
         return -1;
       }
     }
+  } else if (cfg->model == ORC_VAP) {
+    const int32_t vv = orc_vap_version(st, c);
+    for (int32_t p = 0; p < cfg->P; ++p) v[p] = vv;
   } else if (orc_schedule_rule(cfg, c, st->v_prev, v) != 0) {
     free(v);
     return -1;
@@ -193,6 +247,7 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
   memset(st->delta, 0, (size_t)(st->rows * K) * sizeof(double));
   memset(st->count, 0, (size_t)st->rows * sizeof(int64_t));
   const uint8_t b = (uint8_t)((c - 1) % cfg->F);
+  const double eta = cfg->eta_decay ? cfg->eta / sqrt((double)c) : cfg->eta;
   for (int64_t k = 0; k < st->n_obs; ++k) {
     if (st->mb[k] != b) continue;
     int64_t ui = st->i[k], ij = st->j[k];
@@ -206,8 +261,8 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
     double* dL = st->delta + ui * K;
     double* dR = st->delta + (N + ij) * K;
     for (int64_t q = 0; q < K; ++q) {
-      dL[q] += cfg->eta * (e * Rj[q] - cfg->lambda * Li[q]);
-      dR[q] += cfg->eta * (e * Li[q] - cfg->lambda * Rj[q]);
+      dL[q] += eta * (e * Rj[q] - cfg->lambda * Li[q]);
+      dR[q] += eta * (e * Li[q] - cfg->lambda * Rj[q]);
     }
     st->count[ui] += 1;
     st->count[N + ij] += 1;

@@ -8,8 +8,9 @@
  *
  * What one clock c (1-based) computes, producing table version c:
  *   1. the read version v_p(c) of every worker p (Sec. 2.2 SSP condition;
- *      Sec. 3 formal SSP bound; Sec. 4 READ guarantee and server push),
- *      checked against max(0, c-1-s) <= v_p(c) <= c-1;
+ *      Sec. 3 formal SSP bound; Sec. 4 READ guarantee and server push; or
+ *      the value bound of Sec. 2.1 VAP, see ORC_VAP), checked against
+ *      max(0, c-1-s) <= v_p(c) <= c-1;
  *   2. for every observed entry (i, j) of minibatch b = (c-1) mod F, owned by
  *      worker p = w(i): e = D_ij - L_i . R_j at version v_p(c), and the
  *      Sec. 3.1 updates  dL_i += eta (e R_j - lambda L_i),
@@ -33,7 +34,12 @@
 extern "C" {
 #endif
 
-enum { ORC_SSP_LAZY = 0, ORC_ESSP_EAGER = 1, ORC_EXTERNAL = 2 };
+/* ORC_VAP: every worker reads the stalest version v in [max(0, c-1-s), c-1]
+ * whose in-transit updates X[c-1] - X[v] have max-norm at most
+ * v_c = vap_v0 / sqrt(c) (Sec. 2.1 VAP condition, with the shrinking bound
+ * v_t = v0 / sqrt(t) of the SGD-under-VAP theorem of Sec. 3); version c-1
+ * always qualifies. */
+enum { ORC_SSP_LAZY = 0, ORC_ESSP_EAGER = 1, ORC_EXTERNAL = 2, ORC_VAP = 3 };
 
 typedef struct {
   int64_t n_users;     /* N */
@@ -42,7 +48,7 @@ typedef struct {
   int32_t P;           /* workers */
   int32_t s;           /* staleness bound */
   int32_t F;           /* minibatches per pass; clock c uses b = (c-1) mod F */
-  int32_t model;       /* ORC_SSP_LAZY / ORC_ESSP_EAGER / ORC_EXTERNAL */
+  int32_t model;       /* ORC_SSP_LAZY / ORC_ESSP_EAGER / ORC_EXTERNAL / ORC_VAP */
   int32_t phased;      /* SSP: 1 = seeded per-worker refresh phase, 0 = none */
   uint64_t seed;       /* schedule seed */
   double essp_p;       /* ESSP delay ~ Geometric(essp_p), failures before success */
@@ -51,6 +57,8 @@ typedef struct {
   double eta;          /* step size */
   double lambda;       /* l2 penalty, per observation */
   int32_t keep_all;    /* 1 = keep every version (unbounded history) */
+  double vap_v0;       /* ORC_VAP: initial value bound v0 */
+  int32_t eta_decay;   /* 1 = clock c uses eta / sqrt(c) (the step-size schedule of the Sec. 3 theorems) */
 } orc_config;
 
 typedef struct orc_state orc_state;
@@ -78,6 +86,12 @@ int orc_table(const orc_state* st, int32_t version, double* out);
 /* Objective at `version` over ALL observed entries:
  * sq = sum e^2 (Sec. 5 squared loss), pen = sum [e^2 + lambda(|L_i|^2+|R_j|^2)]. */
 int orc_objective(const orc_state* st, int32_t version, double* sq, double* pen);
+
+/* ORC_VAP: the in-transit max-norms the last clock c compared against its
+ * bound: out[k] = |X[c-1] - X[c-1-k]|_inf for k = 0..s (0 where c-1-k < 0),
+ * and *bound = vap_v0 / sqrt(c).  Returns -1 for other models or before
+ * clock 1. */
+int orc_vap_norms(const orc_state* st, double* out, double* bound);
 
 /* The schedule rule alone, for clock c, given the previous read versions.
  * Used by the schedule tests; orc_clock calls the same function. */

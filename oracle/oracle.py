@@ -18,7 +18,7 @@ _SRC = os.path.join(_HERE, "esspt_oracle.c")
 _LIBDIR = os.path.join(_HERE, "_lib")
 _LIB = os.path.join(_LIBDIR, "libesspt_oracle.so")
 
-MODELS = {"ssp": 0, "essp": 1, "external": 2}
+MODELS = {"ssp": 0, "essp": 1, "external": 2, "vap": 3}
 
 
 def build(force: bool = False) -> str:
@@ -53,6 +53,8 @@ class _Cfg(ctypes.Structure):
         ("eta", ctypes.c_double),
         ("lam", ctypes.c_double),
         ("keep_all", ctypes.c_int32),
+        ("vap_v0", ctypes.c_double),
+        ("eta_decay", ctypes.c_int32),
     ]
 
 
@@ -78,6 +80,8 @@ def _load():
         lib.orc_schedule_rule.restype = ctypes.c_int
         lib.orc_ctr_u64.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64]
         lib.orc_ctr_u64.restype = ctypes.c_uint64
+        lib.orc_vap_norms.argtypes = [P, P, P]
+        lib.orc_vap_norms.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -99,12 +103,14 @@ class OracleConfig:
     eta: float = 0.01
     lam: float = 0.05
     keep_all: bool = False
+    vap_v0: float = 0.0
+    eta_decay: bool = False
 
     def _c(self) -> _Cfg:
         return _Cfg(
             self.n_users, self.n_items, self.K, self.P, self.s, self.F, MODELS[self.model],
             int(self.phased), self.seed & 0xFFFFFFFFFFFFFFFF, self.essp_p, self.essp_max_delay,
-            self.cap, self.eta, self.lam, int(self.keep_all),
+            self.cap, self.eta, self.lam, int(self.keep_all), self.vap_v0, int(self.eta_decay),
         )
 
     @classmethod
@@ -112,7 +118,7 @@ class OracleConfig:
         base = dict(
             n_users=w.n_users, n_items=w.n_items, K=w.K, P=w.P, s=w.s, F=w.F, model=w.model,
             seed=w.sched_seed, essp_p=w.essp_p, essp_max_delay=w.essp_max_delay, cap=w.cap,
-            eta=w.eta, lam=w.lam,
+            eta=w.eta, lam=w.lam, vap_v0=w.vap_v0,
         )
         base.update(kw)
         return cls(**base)
@@ -177,6 +183,14 @@ class Oracle:
             raise ValueError("oracle: staleness bound violated")
         if rc != 0:
             raise MemoryError("oracle: allocation failed")
+
+    def vap_norms(self):
+        """VAP: (|X[c-1] - X[c-1-k]|_inf for k = 0..s, the bound) of the last clock."""
+        out = np.empty(self.cfg.s + 1, dtype=np.float64)
+        b = ctypes.c_double()
+        if _load().orc_vap_norms(self._h, _ptr(out), ctypes.byref(b)) != 0:
+            raise ValueError("oracle: not a VAP run, or no clock has run")
+        return out, b.value
 
     def schedule(self) -> np.ndarray:
         out = np.empty(self.cfg.P, dtype=np.int32)

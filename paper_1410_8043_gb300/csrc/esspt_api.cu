@@ -1,5 +1,6 @@
 // The esspt C-ABI: context, version-ring state machine and launches.
 // Every entry point returns a status; no exception crosses the ABI.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -19,6 +20,7 @@ struct esspt_ctx {
   int32_t* v = nullptr;
   uint32_t* status = nullptr;
   uint32_t* thr = nullptr;
+  uint32_t* vap_norm = nullptr;  // [s+1] VAP in-transit norms of the current clock
   int32_t clock = 0;      // clock in progress (0 = table not initialised)
   bool acc_ready = false; // slot of version `clock` holds version clock-1 + INCs so far
   bool sched_set = false; // ESSPT_EXTERNAL: v_p(clock) supplied
@@ -63,7 +65,8 @@ bool config_ok(const esspt_config* c, std::string* why) {
     return *why = "row_width must be a multiple of 4 in [4, 512]", false;
   if (c->num_workers < 1 || c->num_workers > 65536) return *why = "num_workers must be in [1, 65536]", false;
   if (c->staleness < 0 || c->staleness > (1 << 20)) return *why = "staleness must be in [0, 2^20]", false;
-  if (c->model < ESSPT_SSP_LAZY || c->model > ESSPT_EXTERNAL) return *why = "unknown model", false;
+  if (c->model < ESSPT_SSP_LAZY || c->model > ESSPT_VAP) return *why = "unknown model", false;
+  if (c->model == ESSPT_VAP && !(c->vap_v0 >= 0.0)) return *why = "vap_v0 must be >= 0", false;
   if (c->model == ESSPT_ESSP_EAGER) {
     if (!(c->essp_p > 0.0 && c->essp_p <= 1.0)) return *why = "essp_p must be in (0, 1]", false;
     if (c->essp_max_delay < 0) return *why = "essp_max_delay must be >= 0", false;
@@ -79,7 +82,7 @@ int32_t delay_max(const esspt_config* c) {
 }
 
 struct Carve {
-  size_t ring, v, status, thr, total;
+  size_t ring, v, status, thr, vap, total;
 };
 
 Carve carve(const esspt_config* c) {
@@ -93,6 +96,8 @@ Carve carve(const esspt_config* c) {
   o += 256;
   k.thr = o;
   o += align256(sizeof(uint32_t) * (size_t)(delay_max(c) + 1));
+  k.vap = o;
+  o += c->model == ESSPT_VAP ? align256(sizeof(uint32_t) * (size_t)(c->staleness + 1)) : 0;
   k.total = o;
   return k;
 }
@@ -117,6 +122,13 @@ esspt_status need_schedule(esspt_ctx* c) {
 ScheduleArgs schedule_args(const esspt_ctx* c, int32_t clock);
 
 esspt_status run_schedule(esspt_ctx* c) {
+  if (c->cfg.model == ESSPT_VAP) {
+    // In-transit norms of the candidate versions against version clock-1.
+    const int32_t kmax = std::min(c->s, c->clock - 1);
+    ESSPT_CUDA(c, cudaMemsetAsync(c->vap_norm, 0, sizeof(uint32_t) * (size_t)(c->s + 1), c->st));
+    if (kmax > 0)
+      ESSPT_CUDA(c, launch_vap_norms(c->ring, c->n_rows * c->K, c->nslots, c->clock, kmax, c->vap_norm, c->st));
+  }
   ESSPT_CUDA(c, launch_schedule(schedule_args(c, c->clock), c->st));
   return ESSPT_OK;
 }
@@ -151,6 +163,8 @@ ScheduleArgs schedule_args(const esspt_ctx* c, int32_t clock) {
   a.phased = c->cfg.phased;
   a.dmax = c->dmax;
   a.seed = c->cfg.seed;
+  a.vap_norm = c->vap_norm;
+  a.vap_bound = c->cfg.model == ESSPT_VAP ? c->cfg.vap_v0 / std::sqrt((double)clock) : 0.0;
   return a;
 }
 
@@ -271,6 +285,7 @@ esspt_status esspt_create(const esspt_config* cfg, void* d_workspace, size_t byt
   c->v = reinterpret_cast<int32_t*>(w + k.v);
   c->status = reinterpret_cast<uint32_t*>(w + k.status);
   c->thr = reinterpret_cast<uint32_t*>(w + k.thr);
+  if (cfg->model == ESSPT_VAP) c->vap_norm = reinterpret_cast<uint32_t*>(w + k.vap);
   // ESSP delay thresholds thr[k] = floor((1-p)^k * 2^32): P(delay >= k) = (1-p)^k.
   std::vector<uint32_t> thr((size_t)c->dmax + 1, 0u);
   double q = 1.0;
@@ -579,7 +594,9 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   m.item_cnt = c->item_cnt + (int64_t)b * c->n_items;
   m.eta = eta;
   m.cap = cap;
-  m.do_schedule = c->cfg.model != ESSPT_EXTERNAL;
+  // SSP and ESSP schedules need only the previous read versions, so the merge
+  // computes them; VAP needs version c complete, so it runs after the merge.
+  m.do_schedule = c->cfg.model == ESSPT_SSP_LAZY || c->cfg.model == ESSPT_ESSP_EAGER;
   m.sched = schedule_args(c, c->clock + 1);
   ESSPT_CUDA(c, launch_item_merge(m, c->st));
   c->acc_ready = true;

@@ -45,6 +45,8 @@ struct ScheduleArgs {
   int32_t* v;              // [P] read versions (in: v(c-1), out: v(c))
   uint32_t* status;        // latched error bits
   const uint32_t* thr;     // [dmax+1] ESSP delay thresholds, thr[k] = floor((1-p)^k 2^32)
+  const uint32_t* vap_norm;  // [s+1] VAP: bits of |X[c-1] - X[c-1-k]|_inf (fp32, >= 0)
+  double vap_bound;        // VAP: v0 / sqrt(c)
   int32_t P, c, s, model, phased, dmax;
   uint64_t seed;
 };
@@ -110,6 +112,10 @@ struct ItemMergeArgs {
 
 // Launchers (return the launch error, if any).
 cudaError_t launch_schedule(const ScheduleArgs& a, cudaStream_t st);
+// VAP: norm[k] = bits of max |X[c-1] - X[c-1-k]| over the table, k = 1..kmax
+// (norm must be zero on entry; a NaN difference gives +inf).
+cudaError_t launch_vap_norms(const float* ring, int64_t slot_floats, int32_t nslots, int32_t c, int32_t kmax,
+                             uint32_t* norm, cudaStream_t st);
 cudaError_t launch_copy_rows(float* dst, const float* src, int64_t n_floats, cudaStream_t st);
 cudaError_t launch_get(const float* ring, int64_t n_rows, int32_t K, int32_t nslots, const int32_t* v,
                        int32_t worker, const int32_t* ids, int64_t n, float* out, uint32_t* status,

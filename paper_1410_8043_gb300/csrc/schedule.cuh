@@ -1,7 +1,8 @@
 // The read-version rule v_p(c) of one worker (Sec. 2.2 SSP condition and
-// ESSP; Sec. 3 formal SSP bound; Sec. 4 READ guarantee and server push).
-// Integer-only, so it is bit-exact against any other implementation of the
-// same rule.
+// ESSP; Sec. 3 formal SSP bound; Sec. 4 READ guarantee and server push; the
+// Sec. 2.1 VAP value bound).  SSP and ESSP are integer-only, so they are
+// bit-exact against any other implementation of the same rule; VAP compares
+// fp32 max-norms of the table against its bound.
 #pragma once
 
 #include "internal.h"
@@ -29,6 +30,15 @@ __device__ __forceinline__ void schedule_worker(const ScheduleArgs& a, int32_t p
     int32_t d = 0;
     for (int32_t k = 1; k <= a.dmax; ++k) d += (u < a.thr[k]) ? 1 : 0;
     v = max(max(v, a.c - 1 - d), 0);
+  } else if (a.model == ESSPT_VAP) {
+    // Stalest version in the window whose in-transit max-norm is in bound.
+    v = a.c - 1;
+    for (int32_t k = min(a.s, a.c - 1); k >= 1; --k) {
+      if ((double)__uint_as_float(a.vap_norm[k]) <= a.vap_bound) {
+        v = a.c - 1 - k;
+        break;
+      }
+    }
   }
   // ESSPT_EXTERNAL: v was written by the host; only the check below runs.
   if (v < lo || v > a.c - 1) atomicOr(a.status, kErrStale);

@@ -26,6 +26,72 @@ cudaError_t launch_schedule(const ScheduleArgs& a, cudaStream_t st) {
 }
 
 // ---------------------------------------------------------------------------
+// VAP in-transit norms (Sec. 2.1): for k = 1..kmax, the max over the table of
+// |X[c-1] - X[c-1-k]|, folded per block and combined with an integer atomic
+// max on the bits of the non-negative fp32 value (which orders like the
+// value).  Candidates are taken 8 at a time so that each pass reads X[c-1]
+// once for 8 older versions.
+// ---------------------------------------------------------------------------
+constexpr int kVapBatch = 8;
+
+__device__ __forceinline__ float vap_absdiff_max(float m, float4 a, float4 b) {
+  const float d0 = fabsf(a.x - b.x), d1 = fabsf(a.y - b.y), d2 = fabsf(a.z - b.z), d3 = fabsf(a.w - b.w);
+  // fmaxf drops NaN; a NaN difference must fail the bound, so it becomes +inf.
+  const bool nan = (d0 != d0) || (d1 != d1) || (d2 != d2) || (d3 != d3);
+  return nan ? __int_as_float(0x7f800000) : fmaxf(fmaxf(m, fmaxf(d0, d1)), fmaxf(d2, d3));
+}
+
+__global__ void __launch_bounds__(256) vap_norms_kernel(const float4* __restrict__ ring, int64_t slot4, int32_t nslots,
+                                                        int32_t c, int32_t k0, int32_t nk, uint32_t* __restrict__ norm) {
+  __shared__ float red[kVapBatch][8];
+  float m[kVapBatch];
+#pragma unroll
+  for (int t = 0; t < kVapBatch; ++t) m[t] = 0.f;
+  const float4* cur = ring + (int64_t)((c - 1) % nslots) * slot4;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < slot4; q += stride) {
+    const float4 x = cur[q];
+#pragma unroll
+    for (int t = 0; t < kVapBatch; ++t) {
+      if (t < nk) {
+        const int32_t ver = c - 1 - (k0 + t);
+        m[t] = vap_absdiff_max(m[t], x, ring[(int64_t)(ver % nslots) * slot4 + q]);
+      }
+    }
+  }
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+  for (int t = 0; t < kVapBatch; ++t) {
+    float v = m[t];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+    if (lane == 0) red[t][wid] = v;
+  }
+  __syncthreads();
+  if (threadIdx.x < kVapBatch && (int)threadIdx.x < nk) {
+    float v = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) v = fmaxf(v, red[threadIdx.x][w]);
+    if (v > 0.f) atomicMax(norm + k0 + threadIdx.x, __float_as_uint(v));
+  }
+}
+
+cudaError_t launch_vap_norms(const float* ring, int64_t slot_floats, int32_t nslots, int32_t c, int32_t kmax,
+                             uint32_t* norm, cudaStream_t st) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t slot4 = slot_floats / 4;
+  const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>((slot4 + 255) / 256, (int64_t)sms * 8));
+  for (int32_t k0 = 1; k0 <= kmax; k0 += kVapBatch) {
+    const int32_t nk = std::min(kVapBatch, kmax - k0 + 1);
+    vap_norms_kernel<<<blocks, 256, 0, st>>>(reinterpret_cast<const float4*>(ring), slot4, nslots, c, k0, nk, norm);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+// ---------------------------------------------------------------------------
 // Copy-forward: slot(c) <- slot(c-1) for a range of rows, so that the
 // deltas of clock c can land in place (Clock() merge, Sec. 2.1 / Sec. 4).
 // ---------------------------------------------------------------------------

@@ -18,7 +18,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libesspt.so")
 
 OK, EINVAL, ESTATE, ENOSPC, ESTALE, ECUDA = range(6)
 STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ESTATE: "ESTATE", ENOSPC: "ENOSPC", ESTALE: "ESTALE", ECUDA: "ECUDA"}
-MODELS = {"ssp": 0, "essp": 1, "external": 2}
+MODELS = {"ssp": 0, "essp": 1, "external": 2, "vap": 3}
 
 # Every entry point declared in include/esspt.h.
 EXPORTS = (
@@ -48,6 +48,7 @@ class Config(ctypes.Structure):
         ("essp_p", ctypes.c_double),
         ("seed", ctypes.c_uint64),
         ("stream", ctypes.c_void_p),
+        ("vap_v0", ctypes.c_double),
     ]
 
 
@@ -115,14 +116,15 @@ class Table:
     """A stale-synchronous parameter table on one GPU (one `esspt_ctx`)."""
 
     def __init__(self, n_rows: int, K: int, P: int, s: int, model: str = "ssp", phased: bool = True,
-                 seed: int = 8043, essp_p: float = 0.7, essp_max_delay: int = 3, device=None, stream=None):
+                 seed: int = 8043, essp_p: float = 0.7, essp_max_delay: int = 3, vap_v0: float = 0.0,
+                 device=None, stream=None):
         if not torch.cuda.is_available():
             raise RuntimeError("esspt needs a CUDA device")
         L = lib()
         self.device = torch.device(device if device is not None else "cuda")
         self.stream = stream if stream is not None else torch.cuda.current_stream(self.device)
         self.cfg = Config(n_rows, K, P, s, MODELS[model], int(phased), essp_max_delay, essp_p,
-                          seed & 0xFFFFFFFFFFFFFFFF, ctypes.c_void_p(self.stream.cuda_stream))
+                          seed & 0xFFFFFFFFFFFFFFFF, ctypes.c_void_p(self.stream.cuda_stream), vap_v0)
         self.n_rows, self.K, self.P, self.s, self.model = n_rows, K, P, s, model
         nbytes = L.esspt_workspace_bytes(ctypes.byref(self.cfg))
         if nbytes == 0:
@@ -293,7 +295,7 @@ class Table:
     def for_workload(cls, w, data, partition, **kw) -> "Table":
         """A table for an MF workload (gen.workloads.Workload) with data loaded."""
         t = cls(w.n_users + w.n_items, w.K, w.P, w.s, model=w.model, seed=w.sched_seed, essp_p=w.essp_p,
-                essp_max_delay=w.essp_max_delay, **kw)
+                essp_max_delay=w.essp_max_delay, vap_v0=w.vap_v0, **kw)
         wp, mb = partition
         t.mf_load(data.i, data.j, data.D, mb, wp, w.n_users, w.F)
         t.table_init(np.concatenate([data.L0, data.R0]))

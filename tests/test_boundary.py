@@ -46,17 +46,17 @@ def test_config_struct_layout_matches_c(tmp_path):
     probe = tmp_path / "probe.c"
     probe.write_text(
         '#include <stdio.h>\n#include <stddef.h>\n#include "esspt.h"\n'
-        "int main(void){printf(\"%zu %zu %zu %zu %zu\\n\", sizeof(esspt_config),"
+        "int main(void){printf(\"%zu %zu %zu %zu %zu %zu\\n\", sizeof(esspt_config),"
         " offsetof(esspt_config, essp_p), offsetof(esspt_config, seed), offsetof(esspt_config, stream),"
-        " offsetof(esspt_config, essp_max_delay));return 0;}\n"
+        " offsetof(esspt_config, essp_max_delay), offsetof(esspt_config, vap_v0));return 0;}\n"
     )
     exe = tmp_path / "probe"
     subprocess.check_call(["gcc", "-I", os.path.join(ROOT, "include"), str(probe), "-o", str(exe)])
-    size, o_p, o_seed, o_stream, o_md = map(int, subprocess.check_output([str(exe)]).split())
+    size, o_p, o_seed, o_stream, o_md, o_v0 = map(int, subprocess.check_output([str(exe)]).split())
     C = esspt.Config
     assert ctypes.sizeof(C) == size
     assert C.essp_p.offset == o_p and C.seed.offset == o_seed and C.stream.offset == o_stream
-    assert C.essp_max_delay.offset == o_md
+    assert C.essp_max_delay.offset == o_md and C.vap_v0.offset == o_v0
 
 
 def test_status_codes_match_header():
@@ -67,7 +67,8 @@ def test_status_codes_match_header():
                       ("ESSPT_ENOSPC", esspt.ENOSPC), ("ESSPT_ESTALE", esspt.ESTALE), ("ESSPT_ECUDA", esspt.ECUDA)]:
         assert re.search(rf"\b{name}\s*=\s*{val}\b", src)
     for name, val in esspt.MODELS.items():
-        cname = {"ssp": "ESSPT_SSP_LAZY", "essp": "ESSPT_ESSP_EAGER", "external": "ESSPT_EXTERNAL"}[name]
+        cname = {"ssp": "ESSPT_SSP_LAZY", "essp": "ESSPT_ESSP_EAGER", "external": "ESSPT_EXTERNAL",
+                 "vap": "ESSPT_VAP"}[name]
         assert re.search(rf"\b{cname}\s*=\s*{val}\b", src)
 
 

@@ -28,8 +28,9 @@ def _oracle_from_case(case, cap=None, keep_all=False):
     e = np.array(case["entries"], dtype=np.float64).reshape(-1, 3)
     cfg = OracleConfig(
         n_users=case["n_users"], n_items=case["n_items"], K=case["K"], P=case["P"], s=case["s"],
-        F=case["F"], model="external", eta=case["eta"], lam=case["lambda"],
+        F=case["F"], model=case.get("model", "external"), eta=case["eta"], lam=case["lambda"],
         cap=case.get("cap", 0) if cap is None else cap, keep_all=keep_all,
+        vap_v0=case.get("vap_v0", 0.0), eta_decay=case.get("eta_decay", False),
     )
     return Oracle(
         cfg, e[:, 0].astype(np.int32), e[:, 1].astype(np.int32), e[:, 2].astype(np.float32),
@@ -42,14 +43,24 @@ def _frac_table(rows):
     return np.array([[float(Fraction(x)) for x in r] for r in rows], dtype=np.float64)
 
 
-@pytest.mark.parametrize("name", ["single_entry", "stale_k1", "penalty_k2", "hot_row_cap"])
+@pytest.mark.parametrize(
+    "name", ["single_entry", "stale_k1", "penalty_k2", "hot_row_cap", "vap_single_entry", "eta_decay_single_entry"]
+)
 def test_hand_worked_clocks(name):
-    """Sec. 3.1 update rule, stale reads and the Clock() merge, against hand-worked values."""
+    """Sec. 3.1 update rule, stale reads and the Clock() merge, against hand-worked values.
+
+    Cases with the external model give the schedule; the VAP case must choose
+    it by its value bound, and the others read version c-1 (s = 0)."""
     case = _cases()[name]
     o = _oracle_from_case(case)
     N = case["n_users"]
+    external = case.get("model", "external") == "external"
     for c, v in enumerate(case["schedule"], start=1):
-        o.clock(v_ext=v)
+        if external:
+            o.clock(v_ext=v)
+        else:
+            o.clock()
+            assert list(o.schedule()) == v, (c, list(o.schedule()), v)
         want = case["versions"].get(str(c))
         if want is None:
             continue
@@ -323,3 +334,32 @@ def test_cap_scales_only_hot_rows():
     scale = np.minimum(1.0, 20.0 / np.maximum(n, 1))
     assert (n > 20).sum() >= 3  # the cap binds on item rows
     np.testing.assert_allclose(b.table() - x0, scale[:, None] * (a.table() - x0), rtol=1e-12, atol=1e-15)
+
+
+def _vap_pair(v0, s=3, clocks=8):
+    """A VAP oracle and an external-schedule oracle on the same small problem."""
+    d = make_mf_data(n_users=300, n_items=200, n_obs=6000, K=8, seed=77, truth_rank=4, truth_var=0.25, noise_var=0.1)
+    wp = shard_users(300, 4, 78)
+    mb = minibatch_labels(6000, 3, 79)
+    kw = dict(n_users=300, n_items=200, K=8, P=4, s=s, F=3, eta=0.02, lam=0.05)
+    vap = Oracle(OracleConfig(model="vap", vap_v0=v0, **kw), d.i, d.j, d.D, mb, wp, d.L0, d.R0)
+    ext = Oracle(OracleConfig(model="external", **kw), d.i, d.j, d.D, mb, wp, d.L0, d.R0)
+    return vap, ext, s, clocks
+
+
+@pytest.mark.parametrize("v0,stalest", [(0.0, False), (1e300, True)])
+def test_vap_limits_reduce_to_fixed_schedules(v0, stalest):
+    """VAP (Sec. 2.1) at its two limits: a zero value bound admits no update in
+    transit, which is BSP (v = c-1, the s = 0 read of Sec. 2.2); an unbounded
+    one admits every version in the window, so each clock reads the stalest,
+    max(0, c-1-s).  Both runs must match the external-schedule oracle bit for bit."""
+    vap, ext, s, clocks = _vap_pair(v0)
+    for c in range(1, clocks + 1):
+        want = max(0, c - 1 - s) if stalest else c - 1
+        vap.clock()
+        ext.clock(v_ext=np.full(4, want, np.int32))
+        assert list(vap.schedule()) == [want] * 4, c
+        np.testing.assert_array_equal(vap.table(), ext.table())
+    norms, bound = vap.vap_norms()
+    assert bound == v0 / np.sqrt(clocks)
+    assert norms[0] == 0.0 and (norms[1:] > 0).all()
