@@ -321,8 +321,14 @@ __global__ void __launch_bounds__(256, ESSPT_USERS_MINB) sgd_users_kernel(SgdArg
 #ifndef ESSPT_USERS32_MINB
 #define ESSPT_USERS32_MINB 3
 #endif
-constexpr int kUnit = 16;
-constexpr int32_t kUserCost = 5;
+#ifndef ESSPT_U32_UNIT
+#define ESSPT_U32_UNIT 16
+#endif
+#ifndef ESSPT_U32_USERCOST
+#define ESSPT_U32_USERCOST 5
+#endif
+constexpr int kUnit = ESSPT_U32_UNIT;
+constexpr int32_t kUserCost = ESSPT_U32_USERCOST;
 
 // Rows of 68..128 values (17..32 float4 slices), one slice per lane: the
 // whole warp holds one user's row (lane l owns slice l of L_i and of its
@@ -435,13 +441,13 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
       if (n > kHeavy) continue;
       const float4 Lv = stage[wib][b][0][lane];
       // Lanes past the row end read slice 0 (their staged L is zero), so the
-      // item-row loads need no predicate.
+      // item-row loads need no row-end predicate.
       const float4* Rq = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4 + (on ? lane : 0);
       float4 gL = f4_zero();
       // One step: entries tt .. tt+cnt-1 of the user.  It is compiled twice,
-      // for full steps (cnt = 4, the common case) and for the user's last,
-      // partial one, whose missing entries read a row of the window (any
-      // valid one), get e = 0 and add nothing.
+      // for full steps (cnt = 4, the common case), whose loads need no
+      // predicate, and for the user's last, partial one, whose missing
+      // entries load nothing, get e = 0 and add nothing.
       auto step = [&](auto full_tag, int32_t tt, int32_t cnt) {
         constexpr bool kFull = decltype(full_tag)::value;
         const int w0 = tt - win.W;
@@ -453,7 +459,7 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
           const int src = kFull ? w0 + e4 : min(w0 + e4, 31);
           const int32_t j = __shfl_sync(0xffffffffu, win.cj, src);
           dst[e4] = __shfl_sync(0xffffffffu, win.cdst, src);
-          R[e4] = __ldg(Rq + j * K4);
+          R[e4] = (kFull || e4 < cnt) ? __ldg(Rq + j * K4) : f4_zero();
           p[e4] = dot4(Lv, R[e4]);
         }
         // Transposing butterfly: lanes with bit 4 clear keep entries {0, 1},

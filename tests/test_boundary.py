@@ -104,3 +104,10 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     monkeypatch.setattr(esspt, "LIB_PATH", str(tmp_path / "nope.so"))
     with pytest.raises(RuntimeError):
         esspt.lib()
+
+
+def test_report_module_imports_without_gpu():
+    """The staleness/convergence report is part of the package and imports on a CPU host."""
+    from paper_1410_8043_gb300 import report
+
+    assert callable(report.main) and callable(report.run_workload)
