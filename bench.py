@@ -204,12 +204,15 @@ class FloorModel:
         return 12 * int(self.n[b]) + 8 * w.K * w.n_users + 4 * w.K * (users + items), int(self.n[b])
 
 
-def _vap_launches(w, c):
-    """Kernels VAP adds to clock c: the norms for clock c+1 and its schedule."""
-    if w.model != "vap":
-        return 0
-    kmax = min(w.s, c)
-    return (kmax + 7) // 8 + 1
+def _model_launches(w, c):
+    """Kernels the read model adds to clock c: VAP's norms for clock c+1 (one
+    per 8 candidate versions) and its schedule; the row-granular cache's
+    refresh before the SGD kernels."""
+    if w.model == "vap":
+        return (min(w.s, c) + 7) // 8 + 1
+    if w.model == "ssp_row":
+        return 1
+    return 0
 
 
 def run_gpu(args, w):
@@ -367,9 +370,8 @@ def run_gpu(args, w):
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d // K, "d2h_bytes_per_step": d2h // K},
         # per clock: the SGD kernel and the item merge (which also computes the
         # next schedule), plus the chunk and heavy-merge kernels on minibatches
-        # with heavy users; VAP adds its norm kernel (one per 8 candidate
-        # versions) and the schedule kernel after the merge
-        "gpu_launches": int(sum(2 + 2 * model.heavy[(c - 1) % w.F] + _vap_launches(w, c)
+        # with heavy users, plus the read model's own kernels
+        "gpu_launches": int(sum(2 + 2 * model.heavy[(c - 1) % w.F] + _model_launches(w, c)
                                 for c in range(W + 1, W + K + 1))),
         "clocks": clocks,
         "objective": {"clock": c_final, "sq_loss": sq, "penalised": pen},

@@ -8,6 +8,7 @@
 * mid_essp: the mid data under ESSP (eager push), Geometric(0.7) delays
          clamped to [0, 3].
 * mid_vap: the mid data under the VAP value bound 0.3 / sqrt(c), s=3.
+* mid_row: the mid data under row-granular SSP (per-row cached versions), s=3.
 * large: 10M x 1M, 2B entries, Zipf(1.1) users and items, rank-64 model,
          128 workers, 1/50 per clock, SSP s=4, 20 clocks.
 * sweep: the mid data with s in {0,1,2,4,8} x P in {1,8,64,512} x {SSP, ESSP},
@@ -34,7 +35,7 @@ class Workload:
     P: int
     F: int
     s: int
-    model: str  # "ssp" (lazy pull), "essp" (eager push) or "vap" (value bound)
+    model: str  # "ssp" (lazy pull), "essp" (eager push), "vap" (value bound), "ssp_row" (row cache)
     clocks: int
     eta: float
     lam: float
@@ -105,6 +106,11 @@ WORKLOADS = {
     "mid_vap": Workload(
         "mid_vap", 480_000, 18_000, 100_000_000, K=100, P=32, F=20, s=3, model="vap",
         clocks=40, eta=0.005, lam=0.05, cap=20, data=_MID_DATA, vap_v0=0.3,
+    ),
+    # Row-granular SSP (Sec. 4 client cache, a c_param per row) on the mid data.
+    "mid_row": Workload(
+        "mid_row", 480_000, 18_000, 100_000_000, K=100, P=32, F=20, s=3, model="ssp_row",
+        clocks=40, eta=0.005, lam=0.05, cap=20, data=_MID_DATA,
     ),
     "large": Workload(
         "large", 10_000_000, 1_000_000, 2_000_000_000, K=64, P=128, F=50, s=4,

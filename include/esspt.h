@@ -68,6 +68,18 @@ typedef enum {
    * norm never does.  Each clock reads the s+1 candidate versions once more
    * to compute the norms (the cost the paper names for VAP). */
   ESSPT_VAP = 3,
+  /* SSP with a row-granular cache (Sec. 4 "Ensuring Consistency
+   * Guarantees": each cached row carries its own clock c_param, and the
+   * SSPTable client asks the server for a row only when its copy is too
+   * stale).  Worker p holds row r at its own version V[p][r], none before
+   * the first read.  At clock c a read of row r is served by the cached copy
+   * while V[p][r] >= c-1-s; otherwise (or if r is not cached) the row is
+   * first fetched at version c-1.  All reads of a row in one clock see the
+   * same version.  For esspt_mf_sgd_clock the rows a worker reads are the
+   * user and item rows of its entries in the clock's minibatch.  The cache
+   * never evicts: the workspace holds P * n_rows int32 versions.
+   * v_p(c) as reported by esspt_read_schedule is c-1. */
+  ESSPT_SSP_ROW = 4,
 } esspt_model;
 
 typedef struct {
@@ -109,7 +121,10 @@ esspt_status esspt_table_init(esspt_ctx* ctx, const float* rows);
  * each in [0, n_rows)) of worker `worker`'s read version v_p(c) into
  * `d_out` (device, n*K fp32, row-major).  If `h_version_out` is non-NULL the
  * call synchronises and stores v_p(c) there.  Out-of-range row ids are
- * skipped on the device and reported as ESSPT_EINVAL by esspt_poll(). */
+ * skipped on the device and reported as ESSPT_EINVAL by esspt_poll().
+ * ESSPT_SSP_ROW: each row is read at the worker's cached version of that
+ * row, refreshed first as the model says, and `h_version_out` receives the
+ * oldest version read (c-1 if no row was read). */
 esspt_status esspt_get(esspt_ctx* ctx, int32_t worker, const int32_t* d_row_ids, int64_t n,
                        float* d_out, int32_t* h_version_out);
 

@@ -20,7 +20,12 @@
  *     refreshes as lazily as the value bound allows, i.e. reads the stalest
  *     version inside the staleness window whose in-transit max-norm is at
  *     most v0 / sqrt(c) (the shrinking bound v_t = v0 / sqrt(t) of the
- *     SGD-under-VAP theorem, Sec. 3, with t = c); a NaN norm never qualifies.
+ *     SGD-under-VAP theorem, Sec. 3, with t = c); a NaN norm never qualifies;
+ *   - row-granular SSP (Sec. 4 client cache, one c_param per row): a row not
+ *     in the cache is fetched at the server's newest version, c-1 (the first
+ *     read registers the row); a cached row at version v serves a read at
+ *     clock c while v >= c-1-s (the same bound as above) and is otherwise
+ *     refreshed to c-1.  The cache never evicts.
  */
 #include "esspt_oracle.h"
 
@@ -65,6 +70,7 @@ struct orc_state {
   double* delta;    /* rows * K */
   int64_t* count;   /* rows, entries per row in this clock */
   double* vap_norm; /* s+1, ORC_VAP norms of the last clock */
+  int32_t* rowver;  /* ORC_SSP_ROW: P * rows cached versions, -1 = not held */
   double vap_bound; /* ORC_VAP bound of the last clock */
 };
 
@@ -161,7 +167,8 @@ orc_state* orc_create(const orc_config* cfg, int64_t n_obs, const int32_t* i, co
                       const float* D, const uint8_t* minibatch, const int32_t* user_worker,
                       const float* L0, const float* R0) {
   if (!cfg || cfg->n_users <= 0 || cfg->n_items <= 0 || cfg->K <= 0 || cfg->P <= 0 || cfg->s < 0 ||
-      cfg->F <= 0 || n_obs < 0 || cfg->model < 0 || cfg->model > ORC_VAP || (cfg->model == ORC_VAP && !(cfg->vap_v0 >= 0.0)))
+      cfg->F <= 0 || n_obs < 0 || cfg->model < 0 || cfg->model > ORC_SSP_ROW ||
+      (cfg->model == ORC_VAP && !(cfg->vap_v0 >= 0.0)))
     return NULL;
   orc_state* st = (orc_state*)calloc(1, sizeof(orc_state));
   if (!st) return NULL;
@@ -181,7 +188,13 @@ orc_state* orc_create(const orc_config* cfg, int64_t n_obs, const int32_t* i, co
   st->delta = (double*)calloc((size_t)(st->rows * K), sizeof(double));
   st->count = (int64_t*)calloc((size_t)st->rows, sizeof(int64_t));
   st->vap_norm = (double*)calloc((size_t)cfg->s + 1, sizeof(double));
-  if (!st->tables || !st->v_prev || !st->delta || !st->count || !st->vap_norm) {
+  if (cfg->model == ORC_SSP_ROW) {
+    st->rowver = (int32_t*)malloc((size_t)cfg->P * (size_t)st->rows * sizeof(int32_t));
+    if (st->rowver)
+      for (int64_t x = 0; x < (int64_t)cfg->P * st->rows; ++x) st->rowver[x] = -1;
+  }
+  if (!st->tables || !st->v_prev || !st->delta || !st->count || !st->vap_norm ||
+      (cfg->model == ORC_SSP_ROW && !st->rowver)) {
     orc_destroy(st);
     return NULL;
   }
@@ -201,6 +214,7 @@ void orc_destroy(orc_state* st) {
   free(st->delta);
   free(st->count);
   free(st->vap_norm);
+  free(st->rowver);
   free(st);
 }
 
@@ -234,6 +248,8 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
   } else if (cfg->model == ORC_VAP) {
     const int32_t vv = orc_vap_version(st, c);
     for (int32_t p = 0; p < cfg->P; ++p) v[p] = vv;
+  } else if (cfg->model == ORC_SSP_ROW) {
+    for (int32_t p = 0; p < cfg->P; ++p) v[p] = c - 1;
   } else if (orc_schedule_rule(cfg, c, st->v_prev, v) != 0) {
     free(v);
     return -1;
@@ -248,13 +264,32 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
   memset(st->count, 0, (size_t)st->rows * sizeof(int64_t));
   const uint8_t b = (uint8_t)((c - 1) % cfg->F);
   const double eta = cfg->eta_decay ? cfg->eta / sqrt((double)c) : cfg->eta;
+  if (cfg->model == ORC_SSP_ROW) {
+    /* Refresh every row a worker reads this clock, before any read. */
+    const int32_t lo = c - 1 - cfg->s;
+    for (int64_t k = 0; k < st->n_obs; ++k) {
+      if (st->mb[k] != b) continue;
+      int64_t ui = st->i[k], ij = st->j[k];
+      int32_t* V = st->rowver + (int64_t)st->w[ui] * st->rows;
+      if (V[ui] < 0 || V[ui] < lo) V[ui] = c - 1;
+      if (V[N + ij] < 0 || V[N + ij] < lo) V[N + ij] = c - 1;
+    }
+  }
   for (int64_t k = 0; k < st->n_obs; ++k) {
     if (st->mb[k] != b) continue;
     int64_t ui = st->i[k], ij = st->j[k];
     int32_t p = st->w[ui];
-    const double* x = orc_slot(st, v[p]);
-    const double* Li = x + ui * K;
-    const double* Rj = x + (N + ij) * K;
+    const double* Li;
+    const double* Rj;
+    if (cfg->model == ORC_SSP_ROW) {
+      const int32_t* V = st->rowver + (int64_t)p * st->rows;
+      Li = orc_slot(st, V[ui]) + ui * K;
+      Rj = orc_slot(st, V[N + ij]) + (N + ij) * K;
+    } else {
+      const double* x = orc_slot(st, v[p]);
+      Li = x + ui * K;
+      Rj = x + (N + ij) * K;
+    }
     double dot = 0.0;
     for (int64_t q = 0; q < K; ++q) dot += Li[q] * Rj[q];
     double e = (double)st->D[k] - dot;
@@ -283,6 +318,12 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
 }
 
 int32_t orc_version(const orc_state* st) { return st->version; }
+
+int orc_row_version(const orc_state* st, int32_t p, int64_t r, int32_t* out) {
+  if (st->cfg.model != ORC_SSP_ROW || p < 0 || p >= st->cfg.P || r < 0 || r >= st->rows) return -1;
+  *out = st->rowver[(int64_t)p * st->rows + r];
+  return 0;
+}
 
 int orc_schedule(const orc_state* st, int32_t* v_out) {
   if (st->version < 1) return -1;

@@ -39,7 +39,13 @@ extern "C" {
  * v_c = vap_v0 / sqrt(c) (Sec. 2.1 VAP condition, with the shrinking bound
  * v_t = v0 / sqrt(t) of the SGD-under-VAP theorem of Sec. 3); version c-1
  * always qualifies. */
-enum { ORC_SSP_LAZY = 0, ORC_ESSP_EAGER = 1, ORC_EXTERNAL = 2, ORC_VAP = 3 };
+/* ORC_SSP_ROW: SSP with row-granular lazy refresh (Sec. 4 client cache: each
+ * cached row has its own clock c_param).  Worker p holds row r at version
+ * V[p][r], none before its first read.  At clock c every row the worker
+ * reads (the rows of its entries in this clock's minibatch) is refreshed to
+ * version c-1 if it is not held or V[p][r] < c-1-s, and read at V[p][r];
+ * all reads of a row in one clock see the same version. */
+enum { ORC_SSP_LAZY = 0, ORC_ESSP_EAGER = 1, ORC_EXTERNAL = 2, ORC_VAP = 3, ORC_SSP_ROW = 4 };
 
 typedef struct {
   int64_t n_users;     /* N */
@@ -48,7 +54,7 @@ typedef struct {
   int32_t P;           /* workers */
   int32_t s;           /* staleness bound */
   int32_t F;           /* minibatches per pass; clock c uses b = (c-1) mod F */
-  int32_t model;       /* ORC_SSP_LAZY / ORC_ESSP_EAGER / ORC_EXTERNAL / ORC_VAP */
+  int32_t model;       /* ORC_SSP_LAZY / ORC_ESSP_EAGER / ORC_EXTERNAL / ORC_VAP / ORC_SSP_ROW */
   int32_t phased;      /* SSP: 1 = seeded per-worker refresh phase, 0 = none */
   uint64_t seed;       /* schedule seed */
   double essp_p;       /* ESSP delay ~ Geometric(essp_p), failures before success */
@@ -77,7 +83,8 @@ int orc_clock(orc_state* st, const int32_t* v_ext);
 /* Completed clocks (= newest version). */
 int32_t orc_version(const orc_state* st);
 
-/* Read versions used by the last clock, P entries.  Returns -1 before clock 1. */
+/* Read versions used by the last clock, P entries.  Returns -1 before clock 1.
+ * ORC_SSP_ROW reports c-1 for every worker (its reads are per row). */
 int orc_schedule(const orc_state* st, int32_t* v_out);
 
 /* Copy table version `version` ((N+M)*K doubles).  Returns -1 if not held. */
@@ -92,6 +99,10 @@ int orc_objective(const orc_state* st, int32_t version, double* sq, double* pen)
  * and *bound = vap_v0 / sqrt(c).  Returns -1 for other models or before
  * clock 1. */
 int orc_vap_norms(const orc_state* st, double* out, double* bound);
+
+/* ORC_SSP_ROW: the version worker p holds row r at (after the last clock's
+ * refreshes), -1 if it has never read it.  Returns -1 for other models. */
+int orc_row_version(const orc_state* st, int32_t p, int64_t r, int32_t* out);
 
 /* The schedule rule alone, for clock c, given the previous read versions.
  * Used by the schedule tests; orc_clock calls the same function. */

@@ -18,7 +18,7 @@ _SRC = os.path.join(_HERE, "esspt_oracle.c")
 _LIBDIR = os.path.join(_HERE, "_lib")
 _LIB = os.path.join(_LIBDIR, "libesspt_oracle.so")
 
-MODELS = {"ssp": 0, "essp": 1, "external": 2, "vap": 3}
+MODELS = {"ssp": 0, "essp": 1, "external": 2, "vap": 3, "ssp_row": 4}
 
 
 def build(force: bool = False) -> str:
@@ -82,6 +82,8 @@ def _load():
         lib.orc_ctr_u64.restype = ctypes.c_uint64
         lib.orc_vap_norms.argtypes = [P, P, P]
         lib.orc_vap_norms.restype = ctypes.c_int
+        lib.orc_row_version.argtypes = [P, ctypes.c_int32, ctypes.c_int64, P]
+        lib.orc_row_version.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -191,6 +193,13 @@ class Oracle:
         if _load().orc_vap_norms(self._h, _ptr(out), ctypes.byref(b)) != 0:
             raise ValueError("oracle: not a VAP run, or no clock has run")
         return out, b.value
+
+    def row_version(self, p: int, r: int) -> int:
+        """Row-granular SSP: the version worker p holds row r at (-1: never read)."""
+        out = ctypes.c_int32()
+        if _load().orc_row_version(self._h, p, r, ctypes.byref(out)) != 0:
+            raise ValueError("oracle: not a row-granular run, or bad worker/row")
+        return out.value
 
     def schedule(self) -> np.ndarray:
         out = np.empty(self.cfg.P, dtype=np.int32)

@@ -32,6 +32,9 @@ struct esspt_ctx {
   int32_t *rec_u = nullptr, *rec_j = nullptr, *uoff = nullptr, *item_cnt = nullptr, *worker = nullptr;
   int32_t *item_rep = nullptr, *rec_dst = nullptr;
   float *rec_D = nullptr, *dR = nullptr, *dL = nullptr;
+  int32_t* rowver = nullptr;     // row-granular SSP: [P][n_rows] cached versions, -1 = never read
+  int32_t* user_slot = nullptr;  // row-granular SSP: [n_users] per-clock ring slot of each user row
+  int32_t* rec_row = nullptr;    // row-granular SSP: per-clock ring row of each entry's item row
   int4 *chunk = nullptr, *heavy = nullptr;
   std::vector<int64_t> mb_base, chunk_base, heavy_base;
   cudaEvent_t ev_before = nullptr, ev_after = nullptr;
@@ -65,7 +68,9 @@ bool config_ok(const esspt_config* c, std::string* why) {
     return *why = "row_width must be a multiple of 4 in [4, 512]", false;
   if (c->num_workers < 1 || c->num_workers > 65536) return *why = "num_workers must be in [1, 65536]", false;
   if (c->staleness < 0 || c->staleness > (1 << 20)) return *why = "staleness must be in [0, 2^20]", false;
-  if (c->model < ESSPT_SSP_LAZY || c->model > ESSPT_VAP) return *why = "unknown model", false;
+  if (c->model < ESSPT_SSP_LAZY || c->model > ESSPT_SSP_ROW) return *why = "unknown model", false;
+  if (c->model == ESSPT_SSP_ROW && (double)(c->staleness + 2) * (double)c->n_rows >= 2147483647.0)
+    return *why = "row-granular model: (s+2) * n_rows must be < 2^31", false;
   if (c->model == ESSPT_VAP && !(c->vap_v0 >= 0.0)) return *why = "vap_v0 must be >= 0", false;
   if (c->model == ESSPT_ESSP_EAGER) {
     if (!(c->essp_p > 0.0 && c->essp_p <= 1.0)) return *why = "essp_p must be in (0, 1]", false;
@@ -82,7 +87,7 @@ int32_t delay_max(const esspt_config* c) {
 }
 
 struct Carve {
-  size_t ring, v, status, thr, vap, total;
+  size_t ring, v, status, thr, vap, rowver, total;
 };
 
 Carve carve(const esspt_config* c) {
@@ -98,6 +103,8 @@ Carve carve(const esspt_config* c) {
   o += align256(sizeof(uint32_t) * (size_t)(delay_max(c) + 1));
   k.vap = o;
   o += c->model == ESSPT_VAP ? align256(sizeof(uint32_t) * (size_t)(c->staleness + 1)) : 0;
+  k.rowver = o;
+  o += c->model == ESSPT_SSP_ROW ? align256(sizeof(int32_t) * (size_t)c->num_workers * (size_t)c->n_rows) : 0;
   k.total = o;
   return k;
 }
@@ -179,14 +186,14 @@ bool is_host_ptr(const void* p) {
 
 struct MfCarve {
   size_t rec_u, rec_j, rec_D, rec_dst, uoff, mb_base, item_cnt, item_rep, dR, worker, chunk, chunk_base, heavy, heavy_base, dL,
-      total;
+      user_slot, rec_row, total;
   int64_t max_chunks, max_heavy, dR_rows, dL_rows;
 };
 
 // Persistent MF workspace: entries laid out by (minibatch, user), per-minibatch
 // user offsets and item counts, item replica rows, heavy-user lists and the
 // zero-initialised delta replicas dR (items) and dL (heavy users).
-MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int32_t K) {
+MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int32_t K, bool row_mode) {
   MfCarve k{};
   k.max_chunks = layout_max_chunks(n_obs, F);
   k.max_heavy = layout_max_heavy(n_obs, F);
@@ -214,6 +221,10 @@ MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int
   k.heavy = take(sizeof(int4) * k.max_heavy);
   k.heavy_base = take(sizeof(int64_t) * (F + 1));
   k.dL = take(sizeof(float) * (size_t)k.dL_rows * K);
+  // Row-granular SSP: per-clock user slots and entry ring rows (a minibatch
+  // holds at most n_obs entries).
+  k.user_slot = row_mode ? take(sizeof(int32_t) * n_users) : o;
+  k.rec_row = row_mode ? take(sizeof(int32_t) * (n_obs + 4)) : o;
   k.total = o;
   return k;
 }
@@ -286,6 +297,7 @@ esspt_status esspt_create(const esspt_config* cfg, void* d_workspace, size_t byt
   c->status = reinterpret_cast<uint32_t*>(w + k.status);
   c->thr = reinterpret_cast<uint32_t*>(w + k.thr);
   if (cfg->model == ESSPT_VAP) c->vap_norm = reinterpret_cast<uint32_t*>(w + k.vap);
+  if (cfg->model == ESSPT_SSP_ROW) c->rowver = reinterpret_cast<int32_t*>(w + k.rowver);
   // ESSP delay thresholds thr[k] = floor((1-p)^k * 2^32): P(delay >= k) = (1-p)^k.
   std::vector<uint32_t> thr((size_t)c->dmax + 1, 0u);
   double q = 1.0;
@@ -320,6 +332,8 @@ esspt_status esspt_table_init(esspt_ctx* c, const float* rows) {
   if (!rows) return fail(c, ESSPT_EINVAL, "null rows");
   ESSPT_CUDA(c, cudaMemcpyAsync(c->ring, rows, (size_t)c->n_rows * c->K * sizeof(float), cudaMemcpyDefault, c->st));
   ESSPT_CUDA(c, cudaMemsetAsync(c->v, 0, sizeof(int32_t) * c->P, c->st));
+  if (c->rowver)  // no row cached: every byte 0xff is version -1
+    ESSPT_CUDA(c, cudaMemsetAsync(c->rowver, 0xff, sizeof(int32_t) * (size_t)c->P * (size_t)c->n_rows, c->st));
   c->clock = 1;
   c->acc_ready = false;
   c->sched_set = false;
@@ -352,10 +366,15 @@ esspt_status esspt_get(esspt_ctx* c, int32_t worker, const int32_t* d_row_ids, i
   if ((s = need_schedule(c)) != ESSPT_OK) return s;
   if (worker < 0 || worker >= c->P) return fail(c, ESSPT_EINVAL, "worker out of range");
   if (n < 0 || (n > 0 && (!d_row_ids || !d_out))) return fail(c, ESSPT_EINVAL, "bad row list");
-  ESSPT_CUDA(c, launch_get(c->ring, c->n_rows, c->K, c->nslots, c->v, worker, d_row_ids, n, d_out, c->status, c->st));
+  int32_t* vmin = reinterpret_cast<int32_t*>(c->status) + kGetMinWord;
+  if (c->rowver) ESSPT_CUDA(c, cudaMemsetAsync(vmin, 0x7f, sizeof(int32_t), c->st));
+  ESSPT_CUDA(c, launch_get(c->ring, c->n_rows, c->K, c->nslots, c->v, worker, d_row_ids, n, d_out, c->status,
+                           c->rowver, c->clock, c->s, vmin, c->st));
   if (h_version_out) {
-    ESSPT_CUDA(c, cudaMemcpyAsync(h_version_out, c->v + worker, sizeof(int32_t), cudaMemcpyDeviceToHost, c->st));
+    const int32_t* src = c->rowver ? vmin : c->v + worker;
+    ESSPT_CUDA(c, cudaMemcpyAsync(h_version_out, src, sizeof(int32_t), cudaMemcpyDeviceToHost, c->st));
     ESSPT_CUDA(c, cudaStreamSynchronize(c->st));
+    if (c->rowver && *h_version_out == 0x7f7f7f7f) *h_version_out = c->clock - 1;  // no row read
   }
   return ESSPT_OK;
 }
@@ -414,7 +433,7 @@ esspt_status esspt_read_table(esspt_ctx* c, int32_t version, float* out) {
 
 size_t esspt_mf_workspace_bytes(const esspt_ctx* c, int64_t n_obs, int64_t n_users, int32_t F) {
   if (!mf_sizes_ok(c, n_obs, n_users, F)) return 0;
-  return mf_carve(n_obs, n_users, c->n_rows - n_users, F, c->K).total;
+  return mf_carve(n_obs, n_users, c->n_rows - n_users, F, c->K, c->rowver != nullptr).total;
 }
 
 size_t esspt_mf_scratch_bytes(const esspt_ctx* c, int64_t n_obs, int64_t n_users, int32_t F) {
@@ -432,7 +451,7 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   if ((reinterpret_cast<uintptr_t>(d_ws) & 255u) || (reinterpret_cast<uintptr_t>(d_scratch) & 255u))
     return fail(c, ESSPT_EINVAL, "MF buffers must be 256-byte aligned");
   const int64_t n_items = c->n_rows - n_users;
-  const MfCarve k = mf_carve(n_obs, n_users, n_items, F, c->K);
+  const MfCarve k = mf_carve(n_obs, n_users, n_items, F, c->K, c->rowver != nullptr);
   if (bytes < k.total) return fail(c, ESSPT_ENOSPC, "MF workspace too small");
   if (scratch_bytes < layout_scratch_bytes(n_obs, n_users, n_items, F))
     return fail(c, ESSPT_ENOSPC, "MF scratch too small");
@@ -504,6 +523,10 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   c->rec_j = b.rec_j;
   c->rec_D = b.rec_D;
   c->uoff = b.uoff;
+  if (c->rowver) {
+    c->user_slot = reinterpret_cast<int32_t*>(w + k.user_slot);
+    c->rec_row = reinterpret_cast<int32_t*>(w + k.rec_row);
+  }
   c->item_cnt = b.item_cnt;
   c->worker = worker;
   c->item_rep = b.item_rep;
@@ -552,6 +575,28 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   a.lambda = lambda;
   a.cap = cap;
   a.sq_loss = d_sq_loss;
+  if (c->rowver) {
+    // Row-granular SSP: refresh the rows read this clock; the kernels then
+    // take each user's slot and each entry's item ring row from the refresh.
+    RowRefreshArgs r{};
+    r.rowver = c->rowver;
+    r.worker = c->worker;
+    r.uoff = a.uoff;
+    r.rec_u = c->rec_u + c->mb_base[b];
+    r.rec_j = a.rec_j;
+    r.n_rows = c->n_rows;
+    r.n_users = a.n_users;
+    r.n_b = a.n_b;
+    r.c = c->clock;
+    r.s = c->s;
+    r.nslots = c->nslots;
+    r.user_slot = c->user_slot;
+    r.rec_row = c->rec_row;
+    ESSPT_CUDA(c, launch_row_refresh(r, c->st));
+    a.row_mode = 1;
+    a.user_slot = c->user_slot;
+    a.rec_j = c->rec_row;
+  }
   const int64_t nch = c->chunk_base[b + 1] - c->chunk_base[b];
   const int64_t nhv = c->heavy_base[b + 1] - c->heavy_base[b];
   if (c->ev_before) ESSPT_CUDA(c, cudaEventRecord(c->ev_before, c->st));
@@ -596,7 +641,7 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   m.cap = cap;
   // SSP and ESSP schedules need only the previous read versions, so the merge
   // computes them; VAP needs version c complete, so it runs after the merge.
-  m.do_schedule = c->cfg.model == ESSPT_SSP_LAZY || c->cfg.model == ESSPT_ESSP_EAGER;
+  m.do_schedule = c->cfg.model == ESSPT_SSP_LAZY || c->cfg.model == ESSPT_ESSP_EAGER || c->cfg.model == ESSPT_SSP_ROW;
   m.sched = schedule_args(c, c->clock + 1);
   ESSPT_CUDA(c, launch_item_merge(m, c->st));
   c->acc_ready = true;

@@ -15,6 +15,10 @@ enum : uint32_t {
   kErrInput = 4u,     // an MF input index outside its range
 };
 
+// Word of the context's status block (after the error bits) that receives
+// the oldest row version a row-granular GET read.
+constexpr int kGetMinWord = 16;
+
 // Counter-generator stream ids of the schedule.
 constexpr uint64_t kStreamPhase = 101u;
 constexpr uint64_t kStreamDelay = 102u;
@@ -64,7 +68,8 @@ struct SgdArgs {
   const int32_t* v;         // [P] read versions
   const int32_t* worker;    // [n_users]
   const int32_t* uoff;      // [n_users+1] entry offsets of minibatch b (relative)
-  const int32_t* rec_j;     // item of each entry of minibatch b
+  const int32_t* rec_j;     // item of each entry of minibatch b; in row mode the ring row
+                            // (slot * n_rows + N + item) of the item's cached version
   const float* rec_D;       // value of each entry of minibatch b
   const int32_t* rec_dst;   // replica row in dR that each entry's item update adds into
   const int32_t* item_rep;  // [M+1] first replica row of each item in dR
@@ -73,6 +78,8 @@ struct SgdArgs {
   float eta, lambda;
   int32_t cap;
   double* sq_loss;          // optional
+  int32_t row_mode;         // row-granular SSP: per-user slots and per-entry ring rows
+  const int32_t* user_slot; // [n_users] row mode: ring slot of each user's cached row
 };
 
 // Chunks of heavy users: x = user, y = begin, z = end (relative), w = replica row in dL.
@@ -117,12 +124,31 @@ cudaError_t launch_schedule(const ScheduleArgs& a, cudaStream_t st);
 cudaError_t launch_vap_norms(const float* ring, int64_t slot_floats, int32_t nslots, int32_t c, int32_t kmax,
                              uint32_t* norm, cudaStream_t st);
 cudaError_t launch_copy_rows(float* dst, const float* src, int64_t n_floats, cudaStream_t st);
+// GET; with rowver non-null (row-granular SSP at clock c) each row is read at
+// the worker's cached version, refreshed to c-1 first where it is missing or
+// older than c-1-s, and *vmin receives the oldest version read.
 cudaError_t launch_get(const float* ring, int64_t n_rows, int32_t K, int32_t nslots, const int32_t* v,
                        int32_t worker, const int32_t* ids, int64_t n, float* out, uint32_t* status,
-                       cudaStream_t st);
+                       int32_t* rowver, int32_t c, int32_t s, int32_t* vmin, cudaStream_t st);
 cudaError_t launch_inc(float* slot, int64_t n_rows, int32_t K, const int32_t* ids, const float* d, int64_t n,
                        uint32_t* status, cudaStream_t st);
 cudaError_t launch_sgd_users(const SgdArgs& a, cudaStream_t st);
+// Row-granular SSP, before the SGD kernels of clock c: refresh the cached
+// version of every row a worker reads (rowver[p * n_rows + r], -1 = never
+// read) to c-1 where it is missing or older than c-1-s, and write the ring
+// slot of each user's row and the ring row of each entry's item row.
+struct RowRefreshArgs {
+  int32_t* rowver;
+  const int32_t* worker;   // [n_users]
+  const int32_t* uoff;     // [n_users+1] of minibatch b
+  const int32_t* rec_u;    // [n_b] user of each entry
+  const int32_t* rec_j;    // [n_b] item of each entry
+  int64_t n_rows;
+  int32_t n_users, n_b, c, s, nslots;
+  int32_t* user_slot;      // out [n_users]
+  int32_t* rec_row;        // out [n_b]
+};
+cudaError_t launch_row_refresh(const RowRefreshArgs& a, cudaStream_t st);
 cudaError_t launch_sgd_chunks(const ChunkArgs& a, cudaStream_t st);
 cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st);
 cudaError_t launch_item_merge(const ItemMergeArgs& a, cudaStream_t st);

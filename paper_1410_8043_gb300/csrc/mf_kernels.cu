@@ -54,6 +54,12 @@ __device__ __forceinline__ float cap_scale(int32_t cap, int32_t n) {
 // common path.
 __device__ __noinline__ float capped_scale(int32_t cap, int32_t n) { return (float)cap / (float)n; }
 
+// Ring slot of user u's read version: its worker's version, or in
+// row-granular mode the slot its cached row was refreshed to this clock.
+__device__ __forceinline__ int32_t user_slot(const SgdArgs& a, int64_t u) {
+  return a.row_mode ? __ldg(a.user_slot + u) : __ldg(a.v + __ldg(a.worker + u)) % a.nslots;
+}
+
 // Entry t of the minibatch: item, value and the replica row its item update
 // adds into; zeros past the end.
 __device__ __forceinline__ void load_entry(const SgdArgs& a, int32_t t, int32_t& j, float& d, int32_t& dst) {
@@ -113,7 +119,7 @@ __device__ __forceinline__ void process_entries(const SgdArgs& a, const Window<G
   float d[U], part[U];
 #pragma unroll
   for (int u = 0; u < U; ++u) {
-    const float4* row = Rq + __shfl_sync(gmask, win.cj, i + u, G) * K4;
+    const float4* row = Rq + (int64_t)__shfl_sync(gmask, win.cj, i + u, G) * K4;
 #pragma unroll
     for (int t = 0; t < NV; ++t) R[u][t] = act[t] ? __ldg(row + t * G) : f4_zero();
   }
@@ -247,7 +253,7 @@ __global__ void __launch_bounds__(256, ESSPT_USERS_MINB) sgd_users_kernel(SgdArg
     if (uu < a.n_users) {
       m_beg = __ldg(a.uoff + uu);
       m_end = __ldg(a.uoff + uu + 1);
-      m_vs = __ldg(a.v + __ldg(a.worker + uu)) % a.nslots;
+      m_vs = user_slot(a, uu);
     }
     const int64_t g0 = u0 + (int64_t)grp * G;
     const int32_t nusers = (int32_t)max((int64_t)0, min((int64_t)G, (int64_t)a.n_users - g0));
@@ -306,7 +312,7 @@ __global__ void __launch_bounds__(256, ESSPT_USERS_MINB) sgd_users_kernel(SgdArg
 #pragma unroll
       for (int k = 0; k < NV; ++k) gL[k] = f4_zero();
       if (n > 0) {
-        const float4* Rq = ringq + (int64_t)vs * slot4 + (int64_t)a.n_users * K4;
+        const float4* Rq = a.row_mode ? ringq : ringq + (int64_t)vs * slot4 + (int64_t)a.n_users * K4;
         process_range<G, NV>(a, win, beg, end, Lv, gL, Rq, dRq, act, glane, gmask, K4, loss);
       }
       const float sc = a.eta * cap_scale(a.cap, n);
@@ -400,7 +406,7 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
       if (uu < ub) {
         m_beg = __ldg(a.uoff + uu);
         m_end = __ldg(a.uoff + uu + 1);
-        m_vs = __ldg(a.v + __ldg(a.worker + uu)) % a.nslots;
+        m_vs = user_slot(a, uu);
       }
     }
   };
@@ -442,7 +448,8 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
       const float4 Lv = stage[wib][b][0][lane];
       // Lanes past the row end read slice 0 (their staged L is zero), so the
       // item-row loads need no row-end predicate.
-      const float4* Rq = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4 + (on ? lane : 0);
+      const float4* Rq =
+          (a.row_mode ? ring4 : ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4) + (on ? lane : 0);
       float4 gL = f4_zero();
       // One step: entries tt .. tt+cnt-1 of the user.  It is compiled twice,
       // for full steps (cnt = 4, the common case), whose loads need no
@@ -459,7 +466,7 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
           const int src = kFull ? w0 + e4 : min(w0 + e4, 31);
           const int32_t j = __shfl_sync(0xffffffffu, win.cj, src);
           dst[e4] = __shfl_sync(0xffffffffu, win.cdst, src);
-          R[e4] = (kFull || e4 < cnt) ? __ldg(Rq + j * K4) : f4_zero();
+          R[e4] = (kFull || e4 < cnt) ? __ldg(Rq + (int64_t)j * K4) : f4_zero();
           p[e4] = dot4(Lv, R[e4]);
         }
         // Transposing butterfly: lanes with bit 4 clear keep entries {0, 1},
@@ -517,6 +524,39 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
   flush_loss(a.sq_loss, loss, lane);
 }
 
+// Row-granular SSP (Sec. 4 client cache, a clock c_param per cached row):
+// thread x refreshes user x's row (if the user has entries) and entry x's
+// item row in the cache of the reading worker.  All threads that refresh one
+// (worker, row) in a clock write the same value, c-1, so the races are
+// benign and every read of the row in the clock sees one version.
+__global__ void __launch_bounds__(256) row_refresh_kernel(RowRefreshArgs a) {
+  const int32_t lo = a.c - 1 - a.s;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t n = max((int64_t)a.n_users, (int64_t)a.n_b);
+  for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
+    if (x < a.n_users) {
+      int32_t* V = a.rowver + (int64_t)__ldg(a.worker + x) * a.n_rows + x;
+      int32_t v = *V;
+      if (__ldg(a.uoff + x + 1) > __ldg(a.uoff + x) && (v < 0 || v < lo)) {
+        v = a.c - 1;
+        *V = v;
+      }
+      a.user_slot[x] = v < 0 ? 0 : v % a.nslots;
+    }
+    if (x < a.n_b) {
+      const int32_t j = __ldg(a.rec_j + x);
+      const int64_t r = (int64_t)a.n_users + j;
+      int32_t* V = a.rowver + (int64_t)__ldg(a.worker + __ldg(a.rec_u + x)) * a.n_rows + r;
+      int32_t v = *V;
+      if (v < 0 || v < lo) {
+        v = a.c - 1;
+        *V = v;
+      }
+      a.rec_row[x] = (int32_t)((int64_t)(v % a.nslots) * a.n_rows + r);
+    }
+  }
+}
+
 // Chunks of at most kChunk entries of users with more than kHeavy entries:
 // the chunk's partial user update sum (e R - lambda L) goes, unscaled, into
 // one of its user's replica rows of dL; item updates as in the user kernel.
@@ -541,7 +581,7 @@ __global__ void __launch_bounds__(256) sgd_chunks_kernel(ChunkArgs c) {
     const int64_t k = kb + lane / G;
     if (k < c.n_chunks) {
       const int4 ch = c.chunk[k];
-      const int32_t vs = __ldg(a.v + __ldg(a.worker + ch.x)) % a.nslots;
+      const int32_t vs = user_slot(a, ch.x);
       const float4* Lrow = ring4 + (int64_t)vs * slot4 + (int64_t)ch.x * K4;
       float4 Lv[NV], gL[NV];
 #pragma unroll
@@ -552,7 +592,7 @@ __global__ void __launch_bounds__(256) sgd_chunks_kernel(ChunkArgs c) {
       }
       Window<G> win;
       win.reload(a, ch.y, glane);
-      const float4* Rq = ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4 + glane;
+      const float4* Rq = (a.row_mode ? ring4 : ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4) + glane;
       process_range<G, NV>(a, win, ch.y, ch.z, Lv, gL, Rq, dR4 + glane, act, glane, gmask, K4, loss);
 #pragma unroll
       for (int t = 0; t < NV; ++t) {
@@ -694,6 +734,13 @@ cudaError_t launch_sgd_users(const SgdArgs& a, cudaStream_t st) {
   return dispatch_k<UsersF>(a.K, a, st);
 }
 cudaError_t launch_sgd_chunks(const ChunkArgs& c, cudaStream_t st) { return dispatch_k<ChunksF>(c.a.K, c, st); }
+
+cudaError_t launch_row_refresh(const RowRefreshArgs& a, cudaStream_t st) {
+  const int64_t n = std::max<int64_t>(a.n_users, a.n_b);
+  if (n <= 0) return cudaSuccess;
+  row_refresh_kernel<<<grid_for(n, 256, 8), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st) {
   if (a.n_heavy <= 0) return cudaSuccess;

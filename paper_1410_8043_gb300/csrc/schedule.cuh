@@ -30,6 +30,10 @@ __device__ __forceinline__ void schedule_worker(const ScheduleArgs& a, int32_t p
     int32_t d = 0;
     for (int32_t k = 1; k <= a.dmax; ++k) d += (u < a.thr[k]) ? 1 : 0;
     v = max(max(v, a.c - 1 - d), 0);
+  } else if (a.model == ESSPT_SSP_ROW) {
+    // Reads are per row (the row refresh); the worker's nominal version is
+    // the newest one it may read.
+    v = a.c - 1;
   } else if (a.model == ESSPT_VAP) {
     // Stalest version in the window whose in-transit max-norm is in bound.
     v = a.c - 1;

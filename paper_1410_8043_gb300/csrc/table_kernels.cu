@@ -128,13 +128,14 @@ cudaError_t launch_copy_rows(float* dst, const float* src, int64_t n_floats, cud
 // ---------------------------------------------------------------------------
 __global__ void get_rows_kernel(const float* __restrict__ ring, int64_t n_rows, int32_t K, int32_t nslots,
                                 const int32_t* __restrict__ v, int32_t worker, const int32_t* __restrict__ ids,
-                                int64_t n, float* __restrict__ out, uint32_t* status) {
+                                int64_t n, float* __restrict__ out, uint32_t* status, int32_t* rowver, int32_t c,
+                                int32_t s, int32_t* vmin) {
   const int lane = threadIdx.x & 31;
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  const int32_t slot = v[worker] % nslots;
   const int32_t K4 = K >> 2;
-  const float4* base = reinterpret_cast<const float4*>(ring + (int64_t)slot * n_rows * K);
+  const int64_t slot4 = n_rows * K4;
+  const int32_t wslot = rowver ? 0 : v[worker] % nslots;
   for (int64_t k = warp; k < n; k += nwarps) {
     const int32_t r = ids[k];
     float4* o = reinterpret_cast<float4*>(out + k * K);
@@ -142,17 +143,35 @@ __global__ void get_rows_kernel(const float* __restrict__ ring, int64_t n_rows, 
       if (lane == 0) atomicOr(status, kErrRowRange);
       continue;
     }
-    const float4* src = base + (int64_t)r * K4;
+    int32_t slot = wslot;
+    if (rowver) {
+      // Row-granular cache: refresh the row to c-1 if it is missing or too
+      // stale (every refresh of it in this clock writes the same value).
+      int32_t ver = 0;
+      if (lane == 0) {
+        int32_t* V = rowver + (int64_t)worker * n_rows + r;
+        ver = *V;
+        if (ver < 0 || ver < c - 1 - s) {
+          ver = c - 1;
+          *V = ver;
+        }
+        atomicMin(vmin, ver);
+      }
+      slot = __shfl_sync(0xffffffffu, ver, 0) % nslots;
+    }
+    const float4* src = reinterpret_cast<const float4*>(ring) + (int64_t)slot * slot4 + (int64_t)r * K4;
     for (int32_t q = lane; q < K4; q += 32) o[q] = src[q];
   }
 }
 
 cudaError_t launch_get(const float* ring, int64_t n_rows, int32_t K, int32_t nslots, const int32_t* v, int32_t worker,
-                       const int32_t* ids, int64_t n, float* out, uint32_t* status, cudaStream_t st) {
+                       const int32_t* ids, int64_t n, float* out, uint32_t* status, int32_t* rowver, int32_t c,
+                       int32_t s, int32_t* vmin, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   const int threads = 256;
   const int blocks = (int)std::min<int64_t>((n * 32 + threads - 1) / threads, 4096);
-  get_rows_kernel<<<blocks, threads, 0, st>>>(ring, n_rows, K, nslots, v, worker, ids, n, out, status);
+  get_rows_kernel<<<blocks, threads, 0, st>>>(ring, n_rows, K, nslots, v, worker, ids, n, out, status, rowver, c, s,
+                                              vmin);
   return cudaGetLastError();
 }
 

@@ -18,7 +18,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libesspt.so")
 
 OK, EINVAL, ESTATE, ENOSPC, ESTALE, ECUDA = range(6)
 STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ESTATE: "ESTATE", ENOSPC: "ENOSPC", ESTALE: "ESTALE", ECUDA: "ECUDA"}
-MODELS = {"ssp": 0, "essp": 1, "external": 2, "vap": 3}
+MODELS = {"ssp": 0, "essp": 1, "external": 2, "vap": 3, "ssp_row": 4}
 
 # Every entry point declared in include/esspt.h.
 EXPORTS = (

@@ -68,7 +68,7 @@ def test_status_codes_match_header():
         assert re.search(rf"\b{name}\s*=\s*{val}\b", src)
     for name, val in esspt.MODELS.items():
         cname = {"ssp": "ESSPT_SSP_LAZY", "essp": "ESSPT_ESSP_EAGER", "external": "ESSPT_EXTERNAL",
-                 "vap": "ESSPT_VAP"}[name]
+                 "vap": "ESSPT_VAP", "ssp_row": "ESSPT_SSP_ROW"}[name]
         assert re.search(rf"\b{cname}\s*=\s*{val}\b", src)
 
 

@@ -34,7 +34,7 @@ def _oracle_from_case(case, cap=None, keep_all=False):
     )
     return Oracle(
         cfg, e[:, 0].astype(np.int32), e[:, 1].astype(np.int32), e[:, 2].astype(np.float32),
-        np.zeros(e.shape[0], np.uint8), np.array(case["user_worker"], np.int32),
+        np.array(case.get("minibatch", [0] * e.shape[0]), np.uint8), np.array(case["user_worker"], np.int32),
         np.array(case["L0"], np.float32), np.array(case["R0"], np.float32),
     )
 
@@ -44,7 +44,9 @@ def _frac_table(rows):
 
 
 @pytest.mark.parametrize(
-    "name", ["single_entry", "stale_k1", "penalty_k2", "hot_row_cap", "vap_single_entry", "eta_decay_single_entry"]
+    "name",
+    ["single_entry", "stale_k1", "penalty_k2", "hot_row_cap", "vap_single_entry", "eta_decay_single_entry",
+     "row_cache_two_workers"],
 )
 def test_hand_worked_clocks(name):
     """Sec. 3.1 update rule, stale reads and the Clock() merge, against hand-worked values.
@@ -64,6 +66,8 @@ def test_hand_worked_clocks(name):
         want = case["versions"].get(str(c))
         if want is None:
             continue
+        for p, r, ver in case.get("row_versions", {}).get(str(c), []):
+            assert o.row_version(p, r) == ver, (c, p, r)
         x = o.table()
         np.testing.assert_allclose(x[:N], _frac_table(want["L"]), rtol=0, atol=case["tol"])
         np.testing.assert_allclose(x[N:], _frac_table(want["R"]), rtol=0, atol=case["tol"])
@@ -363,3 +367,18 @@ def test_vap_limits_reduce_to_fixed_schedules(v0, stalest):
     norms, bound = vap.vap_norms()
     assert bound == v0 / np.sqrt(clocks)
     assert norms[0] == 0.0 and (norms[1:] > 0).all()
+
+
+def test_row_cache_at_s0_is_bsp():
+    """Row-granular SSP (Sec. 4 client cache) with s = 0 must refresh every row
+    it reads to version c-1 each clock: the BSP schedule, bit for bit."""
+    d = make_mf_data(n_users=300, n_items=200, n_obs=6000, K=8, seed=77, truth_rank=4, truth_var=0.25, noise_var=0.1)
+    wp = shard_users(300, 4, 78)
+    mb = minibatch_labels(6000, 3, 79)
+    kw = dict(n_users=300, n_items=200, K=8, P=4, s=0, F=3, eta=0.02, lam=0.05)
+    row = Oracle(OracleConfig(model="ssp_row", **kw), d.i, d.j, d.D, mb, wp, d.L0, d.R0)
+    ext = Oracle(OracleConfig(model="external", **kw), d.i, d.j, d.D, mb, wp, d.L0, d.R0)
+    for c in range(1, 7):
+        row.clock()
+        ext.clock(v_ext=np.full(4, c - 1, np.int32))
+        np.testing.assert_array_equal(row.table(), ext.table())
