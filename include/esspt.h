@@ -77,7 +77,8 @@ typedef enum {
    * first fetched at version c-1.  All reads of a row in one clock see the
    * same version.  For esspt_mf_sgd_clock the rows a worker reads are the
    * user and item rows of its entries in the clock's minibatch.  The cache
-   * never evicts: the workspace holds P * n_rows int32 versions.
+   * never evicts: the workspace holds P * n_rows int32 versions.  The ring
+   * must hold fewer than 2^31 float4 ((s+2) * n_rows * K/4).
    * v_p(c) as reported by esspt_read_schedule is c-1. */
   ESSPT_SSP_ROW = 4,
 } esspt_model;

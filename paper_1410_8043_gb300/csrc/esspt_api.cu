@@ -69,8 +69,11 @@ bool config_ok(const esspt_config* c, std::string* why) {
   if (c->num_workers < 1 || c->num_workers > 65536) return *why = "num_workers must be in [1, 65536]", false;
   if (c->staleness < 0 || c->staleness > (1 << 20)) return *why = "staleness must be in [0, 2^20]", false;
   if (c->model < ESSPT_SSP_LAZY || c->model > ESSPT_SSP_ROW) return *why = "unknown model", false;
-  if (c->model == ESSPT_SSP_ROW && (double)(c->staleness + 2) * (double)c->n_rows >= 2147483647.0)
-    return *why = "row-granular model: (s+2) * n_rows must be < 2^31", false;
+  // The SGD kernels index item rows with 32-bit float4 offsets; in row mode
+  // the offset spans the whole ring.
+  if (c->model == ESSPT_SSP_ROW &&
+      (double)(c->staleness + 2) * (double)c->n_rows * (double)(c->row_width / 4) >= 2147483647.0)
+    return *why = "row-granular model: the ring must hold fewer than 2^31 float4", false;
   if (c->model == ESSPT_VAP && !(c->vap_v0 >= 0.0)) return *why = "vap_v0 must be >= 0", false;
   if (c->model == ESSPT_ESSP_EAGER) {
     if (!(c->essp_p > 0.0 && c->essp_p <= 1.0)) return *why = "essp_p must be in (0, 1]", false;

@@ -119,7 +119,7 @@ __device__ __forceinline__ void process_entries(const SgdArgs& a, const Window<G
   float d[U], part[U];
 #pragma unroll
   for (int u = 0; u < U; ++u) {
-    const float4* row = Rq + (int64_t)__shfl_sync(gmask, win.cj, i + u, G) * K4;
+    const float4* row = Rq + __shfl_sync(gmask, win.cj, i + u, G) * K4;
 #pragma unroll
     for (int t = 0; t < NV; ++t) R[u][t] = act[t] ? __ldg(row + t * G) : f4_zero();
   }
@@ -466,7 +466,7 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
           const int src = kFull ? w0 + e4 : min(w0 + e4, 31);
           const int32_t j = __shfl_sync(0xffffffffu, win.cj, src);
           dst[e4] = __shfl_sync(0xffffffffu, win.cdst, src);
-          R[e4] = (kFull || e4 < cnt) ? __ldg(Rq + (int64_t)j * K4) : f4_zero();
+          R[e4] = (kFull || e4 < cnt) ? __ldg(Rq + j * K4) : f4_zero();
           p[e4] = dot4(Lv, R[e4]);
         }
         // Transposing butterfly: lanes with bit 4 clear keep entries {0, 1},
