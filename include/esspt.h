@@ -213,6 +213,24 @@ esspt_status esspt_mf_load(esspt_ctx* ctx, const int32_t* d_i, const int32_t* d_
  * added to *d_sq_loss.  ESSPT_ESTATE before esspt_mf_load(). */
 esspt_status esspt_mf_sgd_clock(esspt_ctx* ctx, float eta, float lambda, int32_t cap, double* d_sq_loss);
 
+/* Bytes of the work buffer esspt_mf_sgd_clock_sequential() needs:
+ * P * (n_rows - n_users) * K fp32.  0 before esspt_mf_load(). */
+size_t esspt_mf_sequential_work_bytes(const esspt_ctx* ctx);
+
+/* One clock of MF-SGD with read-my-writes inside each worker, the per-entry
+ * SGD of Sec. 3.1 as each worker runs it (Sec. 5): worker p walks its
+ * entries of minibatch b (its users in ascending id, a user's entries in
+ * input order) and reads L_i and R_j from version v_p(c) plus its own
+ * updates of this clock so far; the summed changes of all workers then make
+ * version c as in esspt_mf_sgd_clock() (same cap rule, same loss output,
+ * then CLOCK).  The entries of one worker form one dependent chain, so this
+ * runs one warp per worker: a semantic variant, far slower than the
+ * minibatch clock.  `d_work` (device, 16-byte aligned, caller-owned) must
+ * hold esspt_mf_sequential_work_bytes() bytes; it is cleared by the call.
+ * ESSPT_EINVAL under the row-granular model ESSPT_SSP_ROW. */
+esspt_status esspt_mf_sgd_clock_sequential(esspt_ctx* ctx, float eta, float lambda, int32_t cap,
+                                           double* d_sq_loss, void* d_work, size_t work_bytes);
+
 /* Objective of Sec. 3.1 / Sec. 5 at table version `version` over ALL loaded
  * entries: *h_sq = sum e^2 (squared loss) and
  * *h_pen = sum [e^2 + lambda (|L_i|^2 + |R_j|^2)] (l2-penalised, per entry).

@@ -25,7 +25,11 @@
  *     in the cache is fetched at the server's newest version, c-1 (the first
  *     read registers the row); a cached row at version v serves a read at
  *     clock c while v >= c-1-s (the same bound as above) and is otherwise
- *     refreshed to c-1.  The cache never evicts.
+ *     refreshed to c-1.  The cache never evicts;
+ *   - sequential (read-my-writes) SGD: the order of a worker's entries in a
+ *     clock is not given; users are taken in ascending id and a user's
+ *     entries in input order.  The worker's summed change joins the Clock()
+ *     merge like any other delta.
  */
 #include "esspt_oracle.h"
 
@@ -168,7 +172,7 @@ orc_state* orc_create(const orc_config* cfg, int64_t n_obs, const int32_t* i, co
                       const float* L0, const float* R0) {
   if (!cfg || cfg->n_users <= 0 || cfg->n_items <= 0 || cfg->K <= 0 || cfg->P <= 0 || cfg->s < 0 ||
       cfg->F <= 0 || n_obs < 0 || cfg->model < 0 || cfg->model > ORC_SSP_ROW ||
-      (cfg->model == ORC_VAP && !(cfg->vap_v0 >= 0.0)))
+      (cfg->model == ORC_VAP && !(cfg->vap_v0 >= 0.0)) || (cfg->sequential && cfg->model == ORC_SSP_ROW))
     return NULL;
   orc_state* st = (orc_state*)calloc(1, sizeof(orc_state));
   if (!st) return NULL;
@@ -228,6 +232,8 @@ static int orc_grow(orc_state* st) {
   return 0;
 }
 
+static int orc_sequential_deltas(orc_state* st, const int32_t* v, uint8_t b, double eta);
+
 int orc_clock(orc_state* st, const int32_t* v_ext) {
   const orc_config* cfg = &st->cfg;
   const int64_t K = cfg->K, N = cfg->n_users;
@@ -264,7 +270,12 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
   memset(st->count, 0, (size_t)st->rows * sizeof(int64_t));
   const uint8_t b = (uint8_t)((c - 1) % cfg->F);
   const double eta = cfg->eta_decay ? cfg->eta / sqrt((double)c) : cfg->eta;
-  if (cfg->model == ORC_SSP_ROW) {
+  if (cfg->sequential) {
+    if (orc_sequential_deltas(st, v, b, eta) != 0) {
+      free(v);
+      return -2;
+    }
+  } else if (cfg->model == ORC_SSP_ROW) {
     /* Refresh every row a worker reads this clock, before any read. */
     const int32_t lo = c - 1 - cfg->s;
     for (int64_t k = 0; k < st->n_obs; ++k) {
@@ -275,7 +286,7 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
       if (V[N + ij] < 0 || V[N + ij] < lo) V[N + ij] = c - 1;
     }
   }
-  for (int64_t k = 0; k < st->n_obs; ++k) {
+  for (int64_t k = 0; k < st->n_obs && !cfg->sequential; ++k) {
     if (st->mb[k] != b) continue;
     int64_t ui = st->i[k], ij = st->j[k];
     int32_t p = st->w[ui];
@@ -314,6 +325,73 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
   }
   memcpy(st->v_prev, v, (size_t)cfg->P * sizeof(int32_t));
   free(v);
+  return 0;
+}
+
+/* Sequential SGD of every worker over its entries of minibatch b at clock c:
+ * worker p's view of row r is X[v_p(c)][r] + its own delta of this clock so
+ * far.  Adds each worker's delta and the entry counts into st->delta and
+ * st->count.  Returns -2 on allocation failure. */
+static int orc_sequential_deltas(orc_state* st, const int32_t* v, uint8_t b, double eta) {
+  const orc_config* cfg = &st->cfg;
+  const int64_t K = cfg->K, N = cfg->n_users;
+  /* Entries of minibatch b grouped by user, input order within a user. */
+  int64_t* uoff = (int64_t*)calloc((size_t)N + 1, sizeof(int64_t));
+  double* mine = (double*)calloc((size_t)(st->rows * K), sizeof(double));
+  int32_t* stamp = (int32_t*)malloc((size_t)st->rows * sizeof(int32_t));
+  int64_t* touched = (int64_t*)malloc((size_t)st->rows * sizeof(int64_t));
+  if (!uoff || !mine || !stamp || !touched) {
+    free(uoff), free(mine), free(stamp), free(touched);
+    return -2;
+  }
+  int64_t nb = 0;
+  for (int64_t k = 0; k < st->n_obs; ++k)
+    if (st->mb[k] == b) uoff[st->i[k] + 1] += 1, ++nb;
+  for (int64_t u = 0; u < N; ++u) uoff[u + 1] += uoff[u];
+  int64_t* order = (int64_t*)malloc((size_t)(nb > 0 ? nb : 1) * sizeof(int64_t));
+  int64_t* fill = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+  if (!order || !fill) {
+    free(uoff), free(mine), free(stamp), free(touched), free(order), free(fill);
+    return -2;
+  }
+  memcpy(fill, uoff, (size_t)N * sizeof(int64_t));
+  for (int64_t k = 0; k < st->n_obs; ++k)
+    if (st->mb[k] == b) order[fill[st->i[k]]++] = k;
+  for (int64_t r = 0; r < st->rows; ++r) stamp[r] = -1;
+
+  for (int32_t p = 0; p < cfg->P; ++p) {
+    const double* x = orc_slot(st, v[p]);
+    int64_t nt = 0;
+    for (int64_t u = 0; u < N; ++u) {
+      if (st->w[u] != p) continue;
+      for (int64_t t = uoff[u]; t < uoff[u + 1]; ++t) {
+        const int64_t k = order[t], ij = st->j[k], rj = N + ij;
+        const int64_t rows2[2] = {u, rj};
+        for (int q2 = 0; q2 < 2; ++q2)
+          if (stamp[rows2[q2]] != p) stamp[rows2[q2]] = p, touched[nt++] = rows2[q2];
+        double* mL = mine + u * K;
+        double* mR = mine + rj * K;
+        double dot = 0.0;
+        for (int64_t q = 0; q < K; ++q) dot += (x[u * K + q] + mL[q]) * (x[rj * K + q] + mR[q]);
+        const double e = (double)st->D[k] - dot;
+        for (int64_t q = 0; q < K; ++q) {
+          const double Lq = x[u * K + q] + mL[q], Rq = x[rj * K + q] + mR[q];
+          mL[q] += eta * (e * Rq - cfg->lambda * Lq);
+          mR[q] += eta * (e * Lq - cfg->lambda * Rq);
+        }
+        st->count[u] += 1;
+        st->count[rj] += 1;
+      }
+    }
+    for (int64_t t = 0; t < nt; ++t) {
+      const int64_t r = touched[t];
+      for (int64_t q = 0; q < K; ++q) {
+        st->delta[r * K + q] += mine[r * K + q];
+        mine[r * K + q] = 0.0;
+      }
+    }
+  }
+  free(uoff), free(mine), free(stamp), free(touched), free(order), free(fill);
   return 0;
 }
 

@@ -16,6 +16,9 @@
  *      Sec. 3.1 updates  dL_i += eta (e R_j - lambda L_i),
  *                         dR_j += eta (e L_i - lambda R_j),
  *      both from the same read version (no read-my-writes, Sec. 3 footnote);
+ *      with `sequential` set, each worker instead walks its entries (users in
+ *      ascending id, a user's entries in input order) and reads L_i and R_j
+ *      from its read version plus its own updates of this clock so far;
  *   3. the Clock() merge X[c] = X[c-1] + scale (.) sum of deltas (additive
  *      updates, Sec. 2.1; coalesced per clock, Sec. 4), where scale is 1
  *      unless the hot-row step cap C is on: then row r's summed delta is
@@ -65,6 +68,8 @@ typedef struct {
   int32_t keep_all;    /* 1 = keep every version (unbounded history) */
   double vap_v0;       /* ORC_VAP: initial value bound v0 */
   int32_t eta_decay;   /* 1 = clock c uses eta / sqrt(c) (the step-size schedule of the Sec. 3 theorems) */
+  int32_t sequential;  /* 1 = each worker runs sequential SGD over its entries, seeing its own
+                          updates within the clock (read-my-writes; Sec. 3.1 as run in Sec. 5) */
 } orc_config;
 
 typedef struct orc_state orc_state;

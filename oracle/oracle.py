@@ -55,6 +55,7 @@ class _Cfg(ctypes.Structure):
         ("keep_all", ctypes.c_int32),
         ("vap_v0", ctypes.c_double),
         ("eta_decay", ctypes.c_int32),
+        ("sequential", ctypes.c_int32),
     ]
 
 
@@ -107,12 +108,14 @@ class OracleConfig:
     keep_all: bool = False
     vap_v0: float = 0.0
     eta_decay: bool = False
+    sequential: bool = False
 
     def _c(self) -> _Cfg:
         return _Cfg(
             self.n_users, self.n_items, self.K, self.P, self.s, self.F, MODELS[self.model],
             int(self.phased), self.seed & 0xFFFFFFFFFFFFFFFF, self.essp_p, self.essp_max_delay,
             self.cap, self.eta, self.lam, int(self.keep_all), self.vap_v0, int(self.eta_decay),
+            int(self.sequential),
         )
 
     @classmethod

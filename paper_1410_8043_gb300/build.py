@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libesspt.so")
-SOURCES = ["table_kernels.cu", "mf_kernels.cu", "layout.cu", "esspt_api.cu", "noalloc.cu"]
+SOURCES = ["table_kernels.cu", "mf_kernels.cu", "seq_kernels.cu", "layout.cu", "esspt_api.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

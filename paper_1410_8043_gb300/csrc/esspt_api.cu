@@ -651,6 +651,52 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   return advance(c, m.do_schedule != 0);
 }
 
+size_t esspt_mf_sequential_work_bytes(const esspt_ctx* c) {
+  if (!c || !c->mf) return 0;
+  return sizeof(float) * (size_t)c->P * (size_t)c->n_items * (size_t)c->K;
+}
+
+esspt_status esspt_mf_sgd_clock_sequential(esspt_ctx* c, float eta, float lambda, int32_t cap, double* d_sq_loss,
+                                           void* d_work, size_t work_bytes) {
+  esspt_status s = need_init(c);
+  if (s != ESSPT_OK) return s;
+  if (!c->mf) return fail(c, ESSPT_ESTATE, "no MF data loaded (call esspt_mf_load)");
+  if ((s = need_schedule(c)) != ESSPT_OK) return s;
+  if (cap < 0) return fail(c, ESSPT_EINVAL, "cap must be >= 0");
+  if (c->rowver) return fail(c, ESSPT_EINVAL, "the sequential clock reads whole-table versions; not ESSPT_SSP_ROW");
+  const size_t need = esspt_mf_sequential_work_bytes(c);
+  if (!d_work || (reinterpret_cast<uintptr_t>(d_work) & 15u)) return fail(c, ESSPT_EINVAL, "work must be 16-byte aligned");
+  if (work_bytes < need) return fail(c, ESSPT_ENOSPC, "sequential work buffer too small");
+  const int32_t b = (c->clock - 1) % c->F;
+  SeqArgs a{};
+  a.ring = c->ring;
+  a.n_rows = c->n_rows;
+  a.K = c->K;
+  a.n_users = (int32_t)c->n_users;
+  a.n_items = (int32_t)c->n_items;
+  a.nslots = c->nslots;
+  a.slot_out = c->clock % c->nslots;
+  a.slot_base = c->acc_ready ? a.slot_out : (c->clock - 1) % c->nslots;
+  a.P = c->P;
+  a.v = c->v;
+  a.worker = c->worker;
+  a.uoff = c->uoff + (int64_t)b * (c->n_users + 1);
+  a.rec_j = c->rec_j + c->mb_base[b];
+  a.rec_D = c->rec_D + c->mb_base[b];
+  a.item_cnt = c->item_cnt + (int64_t)b * c->n_items;
+  a.mine = static_cast<float*>(d_work);
+  a.eta = eta;
+  a.lambda = lambda;
+  a.cap = cap;
+  a.sq_loss = d_sq_loss;
+  ESSPT_CUDA(c, cudaMemsetAsync(d_work, 0, need, c->st));
+  if (c->ev_before) ESSPT_CUDA(c, cudaEventRecord(c->ev_before, c->st));
+  ESSPT_CUDA(c, launch_seq_clock(a, c->st));
+  if (c->ev_after) ESSPT_CUDA(c, cudaEventRecord(c->ev_after, c->st));
+  c->acc_ready = true;
+  return advance(c);
+}
+
 esspt_status esspt_mf_objective(esspt_ctx* c, int32_t version, float lambda, double* d_scratch, double* h_sq,
                                 double* h_pen) {
   esspt_status s = need_init(c);

@@ -149,6 +149,25 @@ struct RowRefreshArgs {
   int32_t* rec_row;        // out [n_b]
 };
 cudaError_t launch_row_refresh(const RowRefreshArgs& a, cudaStream_t st);
+
+// Sequential (read-my-writes) SGD of one clock over minibatch b: the users
+// kernel writes every user row of version c, the item merge every item row.
+struct SeqArgs {
+  float* ring;
+  int64_t n_rows;
+  int32_t K, n_users, n_items, nslots, slot_base, slot_out, P;
+  const int32_t* v;         // [P] read versions
+  const int32_t* worker;    // [n_users]
+  const int32_t* uoff;      // [n_users+1] entry offsets of minibatch b
+  const int32_t* rec_j;     // item of each entry of minibatch b
+  const float* rec_D;
+  const int32_t* item_cnt;  // [n_items] entries per item in minibatch b (hot-row cap)
+  float* mine;              // [P][n_items][K] each worker's item changes this clock (zero on entry)
+  float eta, lambda;
+  int32_t cap;
+  double* sq_loss;          // optional
+};
+cudaError_t launch_seq_clock(const SeqArgs& a, cudaStream_t st);
 cudaError_t launch_sgd_chunks(const ChunkArgs& a, cudaStream_t st);
 cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st);
 cudaError_t launch_item_merge(const ItemMergeArgs& a, cudaStream_t st);

@@ -27,6 +27,7 @@ EXPORTS = (
     "esspt_last_error", "esspt_mf_workspace_bytes", "esspt_mf_scratch_bytes", "esspt_mf_load",
     "esspt_mf_sgd_clock", "esspt_mf_objective", "esspt_mf_minibatch_size", "esspt_mf_export_minibatch",
     "esspt_mf_stage_minibatch", "esspt_set_profile_events", "esspt_mf_worker_objective_noalloc",
+    "esspt_mf_sequential_work_bytes", "esspt_mf_sgd_clock_sequential",
 )
 
 
@@ -81,6 +82,8 @@ def lib() -> ctypes.CDLL:
         "esspt_mf_scratch_bytes": (SZ, [P, I64, I64, I32]),
         "esspt_mf_load": (ctypes.c_int, [P, P, P, P, P, I64, P, I64, I32, P, SZ, P, SZ]),
         "esspt_mf_sgd_clock": (ctypes.c_int, [P, ctypes.c_float, ctypes.c_float, I32, P]),
+        "esspt_mf_sequential_work_bytes": (SZ, [P]),
+        "esspt_mf_sgd_clock_sequential": (ctypes.c_int, [P, ctypes.c_float, ctypes.c_float, I32, P, P, SZ]),
         "esspt_mf_objective": (ctypes.c_int, [P, I32, ctypes.c_float, P, P, P]),
         "esspt_mf_minibatch_size": (ctypes.c_int, [P, I32, P]),
         "esspt_mf_export_minibatch": (ctypes.c_int, [P, I32, P, P, P, P]),
@@ -247,6 +250,16 @@ class Table:
     def mf_sgd_clock(self, eta: float, lam: float, cap: int = 0, sq_loss: torch.Tensor | None = None) -> None:
         """esspt_mf_sgd_clock: one fused clock of MF-SGD (+ CLOCK)."""
         self._check(lib().esspt_mf_sgd_clock(self._h, eta, lam, cap, _ptr(sq_loss)))
+
+    def mf_sgd_clock_sequential(self, eta: float, lam: float, cap: int = 0,
+                                sq_loss: torch.Tensor | None = None) -> None:
+        """esspt_mf_sgd_clock_sequential: one clock with read-my-writes SGD inside each worker.
+        The work buffer is allocated here (torch) on first use and kept."""
+        need = lib().esspt_mf_sequential_work_bytes(self._h)
+        if getattr(self, "_seq_work", None) is None or self._seq_work.numel() < need:
+            self._seq_work = torch.empty(max(need, 16), dtype=torch.uint8, device=self.device)
+        self._check(lib().esspt_mf_sgd_clock_sequential(self._h, eta, lam, cap, _ptr(sq_loss),
+                                                        self._seq_work.data_ptr(), self._seq_work.numel()))
 
     def mf_objective(self, version: int, lam: float):
         """esspt_mf_objective: (sum e^2, sum [e^2 + lam(|L_i|^2+|R_j|^2)]) at `version`."""

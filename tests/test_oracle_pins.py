@@ -31,6 +31,7 @@ def _oracle_from_case(case, cap=None, keep_all=False):
         F=case["F"], model=case.get("model", "external"), eta=case["eta"], lam=case["lambda"],
         cap=case.get("cap", 0) if cap is None else cap, keep_all=keep_all,
         vap_v0=case.get("vap_v0", 0.0), eta_decay=case.get("eta_decay", False),
+        sequential=case.get("sequential", False),
     )
     return Oracle(
         cfg, e[:, 0].astype(np.int32), e[:, 1].astype(np.int32), e[:, 2].astype(np.float32),
@@ -46,7 +47,7 @@ def _frac_table(rows):
 @pytest.mark.parametrize(
     "name",
     ["single_entry", "stale_k1", "penalty_k2", "hot_row_cap", "vap_single_entry", "eta_decay_single_entry",
-     "row_cache_two_workers"],
+     "row_cache_two_workers", "sequential_one_worker"],
 )
 def test_hand_worked_clocks(name):
     """Sec. 3.1 update rule, stale reads and the Clock() merge, against hand-worked values.
@@ -382,3 +383,55 @@ def test_row_cache_at_s0_is_bsp():
         row.clock()
         ext.clock(v_ext=np.full(4, c - 1, np.int32))
         np.testing.assert_array_equal(row.table(), ext.table())
+
+
+def _small_seq_problem(n_users, n_items, n_obs, P, F, seed):
+    d = make_mf_data(n_users=n_users, n_items=n_items, n_obs=n_obs, K=8, seed=seed, truth_rank=4, truth_var=0.25,
+                     noise_var=0.1)
+    return d, shard_users(n_users, P, seed + 1), minibatch_labels(n_obs, F, seed + 2)
+
+
+def test_sequential_is_textbook_sgd_for_one_worker():
+    """With one worker, s = 0 and one minibatch, the sequential clock is plain
+    sequential SGD (Sec. 3.1 applied entry by entry, in place): users in
+    ascending id, a user's entries in input order."""
+    d, _, _ = _small_seq_problem(40, 30, 400, 1, 1, 31)
+    wp = np.zeros(40, np.int32)
+    mb = np.zeros(400, np.uint8)
+    eta, lam = 0.03, 0.05
+    o = Oracle(OracleConfig(n_users=40, n_items=30, K=8, P=1, s=0, F=1, model="ssp", eta=eta, lam=lam,
+                            sequential=True), d.i, d.j, d.D, mb, wp, d.L0, d.R0)
+    L = d.L0.astype(np.float64).copy()
+    R = d.R0.astype(np.float64).copy()
+    order = sorted(range(400), key=lambda k: (int(d.i[k]), k))
+    for c in range(1, 4):
+        o.clock()
+        for k in order:
+            u, j = int(d.i[k]), int(d.j[k])
+            e = float(d.D[k]) - float(L[u] @ R[j])
+            gl = eta * (e * R[j] - lam * L[u])
+            gr = eta * (e * L[u] - lam * R[j])
+            L[u] += gl
+            R[j] += gr
+        x = o.table()
+        np.testing.assert_allclose(x[:40], L, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(x[40:], R, rtol=0, atol=1e-12)
+
+
+def test_sequential_equals_minibatch_with_one_entry_per_worker():
+    """If no worker has two entries in a clock, reading one's own writes
+    changes nothing: the sequential and minibatch clocks agree (to the order
+    of the fp64 sums)."""
+    n = 60
+    d, _, _ = _small_seq_problem(n, 20, n, n, 1, 41)
+    i = np.arange(n, dtype=np.int32)  # one entry per user, each user its own worker
+    wp = np.arange(n, dtype=np.int32)
+    mb = np.zeros(n, np.uint8)
+    kw = dict(n_users=n, n_items=20, K=8, P=n, s=2, F=1, model="ssp", phased=True, eta=0.05, lam=0.05)
+    seq = Oracle(OracleConfig(sequential=True, **kw), i, d.j, d.D, mb, wp, d.L0, d.R0)
+    bat = Oracle(OracleConfig(**kw), i, d.j, d.D, mb, wp, d.L0, d.R0)
+    for _ in range(5):
+        seq.clock()
+        bat.clock()
+        np.testing.assert_array_equal(seq.schedule(), bat.schedule())
+        np.testing.assert_allclose(seq.table(), bat.table(), rtol=1e-13, atol=1e-15)
