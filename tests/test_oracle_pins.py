@@ -267,13 +267,18 @@ def test_s0_invariant_to_workers_and_model():
                 np.testing.assert_array_equal(o.table(), ref)
 
 
-@pytest.mark.parametrize("model", ["ssp", "essp"])
-def test_ring_equals_unbounded_history(model):
-    """An (s+2)-slot version ring gives the same tables as keeping every version."""
+@pytest.mark.parametrize(
+    "model,extra",
+    [("ssp", {}), ("essp", {}), ("vap", {"vap_v0": 0.3}), ("ssp_row", {}), ("ssp", {"sequential": True}),
+     ("essp", {"sequential": True})],
+)
+def test_ring_equals_unbounded_history(model, extra):
+    """An (s+2)-slot version ring gives the same tables as keeping every
+    version: no read model ever needs a version outside the ring."""
     d = _small_data()
     P, s, F = 5, 3, 3
     wp, mb = shard_users(d.n_users, P, 2), minibatch_labels(d.n_obs, F, 3)
-    kw = dict(n_users=d.n_users, n_items=d.n_items, K=d.K, P=P, s=s, F=F, model=model, eta=0.02)
+    kw = dict(n_users=d.n_users, n_items=d.n_items, K=d.K, P=P, s=s, F=F, model=model, eta=0.02, **extra)
     a = Oracle(OracleConfig(**kw), d.i, d.j, d.D, mb, wp, d.L0, d.R0)
     b = Oracle(OracleConfig(keep_all=True, **kw), d.i, d.j, d.D, mb, wp, d.L0, d.R0)
     for _ in range(25):
