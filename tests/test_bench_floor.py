@@ -1,0 +1,52 @@
+"""Host logic of bench.py's roofline: the compulsory-bytes model of one clock
+against a brute-force count on a small workload, and the kernel-launch count
+of each read model."""
+import numpy as np
+
+from gen import make_mf_data, minibatch_labels, shard_users
+
+
+def _brute_floor(w, d, wp, mb, c, v):
+    """12 B per entry; 8K bytes per user row (read c-1, write c); 4K bytes per
+    stale user row read and per distinct (item, stale version) read."""
+    b = (c - 1) % w.F
+    idx = np.flatnonzero(mb == b)
+    total = 12 * idx.size + 8 * w.K * w.n_users
+    users = set()
+    items = set()
+    for k in idx:
+        u, j = int(d.i[k]), int(d.j[k])
+        ver = int(v[wp[u]])
+        if ver != c - 1:
+            users.add(u)
+            items.add((j, ver))
+    return total + 4 * w.K * (len(users) + len(items)), idx.size
+
+
+def test_floor_model_matches_brute_force():
+    import bench
+    from gen.workloads import Workload
+
+    d = make_mf_data(n_users=120, n_items=40, n_obs=3000, K=8, seed=5, truth_rank=2)
+    P, F = 4, 3
+    wp = shard_users(120, P, 6)
+    mb = minibatch_labels(3000, F, 7)
+    w = Workload("t", 120, 40, 3000, K=8, P=P, F=F, s=3, model="ssp", clocks=5, eta=0.01, lam=0.05, cap=0)
+    m = bench.FloorModel(w, d, wp, mb)
+    rng = np.random.default_rng(0)
+    for c in range(1, 9):
+        v = rng.integers(max(0, c - 1 - w.s), c, size=P).astype(np.int32)
+        assert m.bytes(c, v) == _brute_floor(w, d, wp, mb, c, v)
+
+
+def test_model_launch_counts():
+    import bench
+    from gen import workload
+
+    assert bench._model_launches(workload("mid"), 10) == 0
+    assert bench._model_launches(workload("mid_essp"), 10) == 0
+    assert bench._model_launches(workload("mid_row"), 10) == 1
+    # VAP: the norms of clock c+1 take one kernel per 8 candidate versions, plus the schedule.
+    w = workload("mid_vap")
+    assert bench._model_launches(w, 1) == 2 and bench._model_launches(w, 10) == 2
+    assert bench._model_launches(w.with_(s=9), 10) == 3
