@@ -76,6 +76,7 @@ struct orc_state {
   double* vap_norm; /* s+1, ORC_VAP norms of the last clock */
   int32_t* rowver;  /* ORC_SSP_ROW: P * rows cached versions, -1 = not held */
   double vap_bound; /* ORC_VAP bound of the last clock */
+  double clock_sq;  /* sum of e^2 over the last clock's entries */
 };
 
 static double* orc_slot(const orc_state* st, int32_t version) {
@@ -268,6 +269,7 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
   /* 2. Deltas of every entry of minibatch b, each at its worker's version. */
   memset(st->delta, 0, (size_t)(st->rows * K) * sizeof(double));
   memset(st->count, 0, (size_t)st->rows * sizeof(int64_t));
+  st->clock_sq = 0.0;
   const uint8_t b = (uint8_t)((c - 1) % cfg->F);
   const double eta = cfg->eta_decay ? cfg->eta / sqrt((double)c) : cfg->eta;
   if (cfg->sequential) {
@@ -304,6 +306,7 @@ int orc_clock(orc_state* st, const int32_t* v_ext) {
     double dot = 0.0;
     for (int64_t q = 0; q < K; ++q) dot += Li[q] * Rj[q];
     double e = (double)st->D[k] - dot;
+    st->clock_sq += e * e;
     double* dL = st->delta + ui * K;
     double* dR = st->delta + (N + ij) * K;
     for (int64_t q = 0; q < K; ++q) {
@@ -374,6 +377,7 @@ static int orc_sequential_deltas(orc_state* st, const int32_t* v, uint8_t b, dou
         double dot = 0.0;
         for (int64_t q = 0; q < K; ++q) dot += (x[u * K + q] + mL[q]) * (x[rj * K + q] + mR[q]);
         const double e = (double)st->D[k] - dot;
+        st->clock_sq += e * e;
         for (int64_t q = 0; q < K; ++q) {
           const double Lq = x[u * K + q] + mL[q], Rq = x[rj * K + q] + mR[q];
           mL[q] += eta * (e * Rq - cfg->lambda * Lq);
@@ -400,6 +404,12 @@ int32_t orc_version(const orc_state* st) { return st->version; }
 int orc_row_version(const orc_state* st, int32_t p, int64_t r, int32_t* out) {
   if (st->cfg.model != ORC_SSP_ROW || p < 0 || p >= st->cfg.P || r < 0 || r >= st->rows) return -1;
   *out = st->rowver[(int64_t)p * st->rows + r];
+  return 0;
+}
+
+int orc_clock_loss(const orc_state* st, double* out) {
+  if (st->version < 1) return -1;
+  *out = st->clock_sq;
   return 0;
 }
 

@@ -99,6 +99,12 @@ int orc_table(const orc_state* st, int32_t version, double* out);
  * sq = sum e^2 (Sec. 5 squared loss), pen = sum [e^2 + lambda(|L_i|^2+|R_j|^2)]. */
 int orc_objective(const orc_state* st, int32_t version, double* sq, double* pen);
 
+/* Squared loss of the last clock: sum of e^2 over the entries of its
+ * minibatch, each e taken where its update was computed (at the worker's
+ * read version; in the sequential variant, at the worker's view just before
+ * the entry).  Returns -1 before clock 1. */
+int orc_clock_loss(const orc_state* st, double* out);
+
 /* ORC_VAP: the in-transit max-norms the last clock c compared against its
  * bound: out[k] = |X[c-1] - X[c-1-k]|_inf for k = 0..s (0 where c-1-k < 0),
  * and *bound = vap_v0 / sqrt(c).  Returns -1 for other models or before

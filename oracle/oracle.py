@@ -83,6 +83,8 @@ def _load():
         lib.orc_ctr_u64.restype = ctypes.c_uint64
         lib.orc_vap_norms.argtypes = [P, P, P]
         lib.orc_vap_norms.restype = ctypes.c_int
+        lib.orc_clock_loss.argtypes = [P, P]
+        lib.orc_clock_loss.restype = ctypes.c_int
         lib.orc_row_version.argtypes = [P, ctypes.c_int32, ctypes.c_int64, P]
         lib.orc_row_version.restype = ctypes.c_int
         _lib = lib
@@ -196,6 +198,13 @@ class Oracle:
         if _load().orc_vap_norms(self._h, _ptr(out), ctypes.byref(b)) != 0:
             raise ValueError("oracle: not a VAP run, or no clock has run")
         return out, b.value
+
+    def clock_loss(self) -> float:
+        """Sum of e^2 over the last clock's entries, each at its read version."""
+        out = ctypes.c_double()
+        if _load().orc_clock_loss(self._h, ctypes.byref(out)) != 0:
+            raise ValueError("oracle: no clock has run")
+        return out.value
 
     def row_version(self, p: int, r: int) -> int:
         """Row-granular SSP: the version worker p holds row r at (-1: never read)."""

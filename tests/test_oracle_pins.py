@@ -77,6 +77,33 @@ def test_hand_worked_clocks(name):
         assert got[0] == float(Fraction(sq)) and got[1] == float(Fraction(pen))
 
 
+@pytest.mark.parametrize("name", ["single_entry", "stale_k1", "penalty_k2", "sequential_one_worker"])
+def test_hand_worked_clock_losses(name):
+    """The clock's own squared loss (sum of e^2 over its entries, each at its
+    read version) against the hand-derived residuals of each clock."""
+    case = _cases()[name]
+    o = _oracle_from_case(case)
+    external = case.get("model", "external") == "external"
+    want = case["clock_loss"]
+    for c, v in enumerate(case["schedule"], start=1):
+        o.clock(v_ext=v) if external else o.clock()
+        if str(c) in want:
+            assert o.clock_loss() == float(Fraction(want[str(c)])), (name, c)
+
+
+def test_clock_loss_full_batch_bsp_is_squared_loss():
+    """With one minibatch (F = 1) and s = 0 every entry is read at X[c-1], so
+    the clock's loss is the squared loss J of version c-1 (Sec. 5)."""
+    d = make_mf_data(n_users=40, n_items=25, n_obs=600, K=6, seed=13, truth_rank=2)
+    P = 3
+    cfg = OracleConfig(n_users=40, n_items=25, K=6, P=P, s=0, F=1, model="essp", eta=0.01, lam=0.05)
+    o = Oracle(cfg, d.i, d.j, d.D, np.zeros(600, np.uint8), shard_users(40, P, 2), d.L0, d.R0)
+    for c in range(1, 5):
+        want = o.objective(c - 1)[0]
+        o.clock()
+        assert o.clock_loss() == pytest.approx(want, rel=1e-12), c
+
+
 def test_bound_violation_rejected():
     """A read that misses updates of clocks <= c-s-1 breaks the SSP condition (Sec. 2.2)."""
     case = _cases()["stale_k1"]
