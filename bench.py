@@ -1,11 +1,14 @@
 """Benchmark: stale-synchronous MF-SGD clocks on GB300 (ratings per second).
 
-One step = one whole clock of the hot path (read-version schedule, Clock()
-copy of the item rows, fused SGD gather/residual/update/merge) over one
-minibatch of the synthetic Netflix-shaped workload (480k x 18k, 100M
-entries, rank 100, 32 workers, SSP s=3, 1/20 of the data per clock).
+One step = one whole clock of the hot path (read-version schedule, fused SGD
+gather/residual/update with the user-row merge, the Clock() merge of the
+item rows) over one minibatch.  The headline workload is the large one
+(10M x 1M, 2B entries, Zipf(1.1) users and items, rank 64, 128 workers,
+SSP s=4, 1/50 of the data per clock); the Netflix-shaped mid workload
+(480k x 18k, 100M entries, rank 100, 32 workers, SSP s=3, 1/20 per clock)
+is measured in the same run and reported under "extra_workloads".
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload mid]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload large] [--extra mid]
     python bench.py --impl reference ...   # the fp64 CPU oracle, same metric
 
 Prints one JSON line.  With N > 1 (torchrun) every rank runs an independent
@@ -171,37 +174,61 @@ class FloorModel:
     versions v): 12 B per entry (i, j, D); the merge of every user row (read
     version c-1, write version c); each user row read at a stale version
     (v != c-1) by a user with entries; each distinct (item, stale version)
-    row read.  Item rows of version c stay in L2 while deltas fold in."""
+    row read.  Item rows of version c-1 count as resident (the previous
+    clock's merge just wrote them).  Counted with torch on `device` (the
+    distinct pairs by sorting), one minibatch at a time."""
 
-    def __init__(self, w, data, wp, mb):
+    def __init__(self, w, data, wp, mb, device="cpu"):
+        import torch
+
         self.w = w
-        P, M = w.P, w.n_items
-        self.n = np.zeros(w.F, np.int64)
-        self.users_of = np.zeros((w.F, P), np.int64)
-        self.items_of = []
-        self.heavy = np.zeros(w.F, bool)
-        for b in range(w.F):
-            idx = np.flatnonzero(mb == b)
-            ui, jj = data.i[idx], data.j[idx]
-            self.n[b] = idx.size
-            # users with more than 96 entries go through two extra kernels
-            self.heavy[b] = idx.size > 0 and np.bincount(ui).max() > 96
-            has = np.zeros(w.n_users, bool)
-            has[ui] = True
-            self.users_of[b] = np.bincount(wp[has], minlength=P)
-            m = np.zeros((P, M), bool)
-            m[wp[ui], jj] = True
-            self.items_of.append(m)
+        self.dev = torch.device(device)
+        self.i = torch.as_tensor(np.ascontiguousarray(data.i)).to(self.dev)
+        self.j = torch.as_tensor(np.ascontiguousarray(data.j)).to(self.dev)
+        self.mb = torch.as_tensor(np.ascontiguousarray(mb)).to(self.dev)
+        self.wp = torch.as_tensor(np.ascontiguousarray(wp)).to(self.dev).long()
+        self._b = None
+        self._per_b = {}
+
+    def _minibatch(self, b):
+        """(entries, worker of each user with entries, distinct worker*M + item
+        pairs, some user has more than 96 entries) of minibatch b."""
+        import torch
+
+        if self._b != b:
+            idx = torch.nonzero(self.mb == b).squeeze(1)
+            ui = self.i[idx].long()
+            jj = self.j[idx].long()
+            users, cnt = torch.unique(ui, return_counts=True)
+            uw = self.wp[users]
+            pj = torch.unique(self.wp[ui] * self.w.n_items + jj)
+            heavy = bool(cnt.numel() and int(cnt.max()) > 96)
+            self._cache = (int(idx.numel()), uw, pj, heavy)
+            self._b = b
+            del idx, ui, jj, users, cnt
+        return self._cache
+
+    def heavy(self, b) -> bool:
+        """Whether minibatch b has a user with more than 96 entries (those go
+        through the chunk and heavy-merge kernels)."""
+        if b not in self._per_b:
+            self._per_b[b] = self._minibatch(b)[3]
+        return self._per_b[b]
 
     def bytes(self, c, v):
+        import torch
+
         w = self.w
         b = (c - 1) % w.F
-        stale = v != (c - 1)
-        users = int(self.users_of[b][stale].sum())
-        items = 0
-        for ver in np.unique(v[stale]):
-            items += int(np.count_nonzero(self.items_of[b][v == ver].any(axis=0)))
-        return 12 * int(self.n[b]) + 8 * w.K * w.n_users + 4 * w.K * (users + items), int(self.n[b])
+        n, uw, pj, heavy = self._minibatch(b)
+        self._per_b[b] = heavy
+        vt = torch.as_tensor(np.ascontiguousarray(v, dtype=np.int64)).to(self.dev)
+        stale = vt != (c - 1)
+        users = int(stale[uw].sum())
+        p = pj // w.n_items
+        sp = stale[p]
+        items = int(torch.unique(vt[p[sp]] * w.n_items + (pj[sp] % w.n_items)).numel())
+        return 12 * n + 8 * w.K * w.n_users + 4 * w.K * (users + items), n
 
 
 def _model_launches(w, c):
@@ -215,29 +242,65 @@ def _model_launches(w, c):
     return 0
 
 
-def run_gpu(args, w):
+def _stage_overlapped(t, w, host_mb, W, K, stream, copy_stream, loss_d, loss_h):
+    """K clocks through the public API with host inputs: minibatch of clock
+    c+1 is copied from pinned host memory on `copy_stream` while clock c runs
+    on `stream`; each clock's squared loss is copied back to pinned host
+    memory.  Returns (h2d bytes, d2h bytes)."""
+    import torch
+
+    F = w.F
+    staged = [torch.cuda.Event() for _ in range(K)]
+    done = [torch.cuda.Event() for _ in range(K)]
+    h2d = d2h = 0
+
+    def stage(k):
+        nonlocal h2d
+        c = W + 1 + k
+        b = (c - 1) % F
+        # minibatch b was last read by clock c - F: wait for it
+        if k - F >= 0:
+            copy_stream.wait_event(done[k - F])
+        u, j, D, uoff = host_mb[b]
+        t.mf_stage_minibatch(b, u, j, D, uoff, stream=copy_stream)
+        staged[k].record(copy_stream)
+        h2d += 4 * (u.numel() + j.numel() + D.numel() + uoff.numel())
+
+    start = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    copy_stream.wait_event(start)
+    stage(0)
+    for k in range(K):
+        if k + 1 < K:
+            stage(k + 1)
+        stream.wait_event(staged[k])
+        t.mf_sgd_clock(w.eta, w.lam, w.cap, sq_loss=loss_d[k:k + 1])
+        with torch.cuda.stream(stream):
+            loss_h[k:k + 1].copy_(loss_d[k:k + 1], non_blocking=True)
+        d2h += 8
+        done[k].record(stream)
+    return start, h2d, d2h
+
+
+def measure(args, w, dev, world, rank, local):
+    """One workload: accounting pass, the timed clocks, the end-to-end clocks.
+    Returns the bench fields of that workload, plus the data for the CPU
+    baseline."""
     import torch
 
     from paper_1410_8043_gb300 import esspt
-
-    world, rank, local = _dist()
-    if world > 1:
-        import torch.distributed as dist
-
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
 
     t0 = time.time()
     data = w.make_data()
     wp, mb = w.partition()
     gen_s = time.time() - t0
     stream = torch.cuda.Stream(dev)
+    t0 = time.time()
     with torch.cuda.stream(stream):
         t = esspt.Table.for_workload(w, data, (wp, mb), device=dev, stream=stream)
+    load_s = time.time() - t0
     x0 = torch.as_tensor(np.concatenate([data.L0, data.R0]), device=dev)
-    model = FloorModel(w, data, wp, mb)
+    model = FloorModel(w, data, wp, mb, device=dev)
 
     K, W = args.steps, args.warmup
     # Accounting pass (untimed): read versions of every clock -> floor bytes.
@@ -253,7 +316,9 @@ def run_gpu(args, w):
             stale += np.bincount(c - 1 - v, minlength=w.s + 1)[: w.s + 1]
         t.mf_sgd_clock(w.eta, w.lam, w.cap)
     t.poll()
-    sq0, pen0 = None, None
+    heavy = {b: model.heavy(b) for b in {(c - 1) % w.F for c in range(W + 1, W + K + 1)}}
+    del model
+    torch.cuda.empty_cache()
 
     # Timed run from version 0 again.
     t.table_init(x0)
@@ -290,30 +355,25 @@ def run_gpu(args, w):
     c_final = t.clock_index - 1
     sq, pen = t.mf_objective(c_final, w.lam)
 
-    # End to end through the public API: each step copies its minibatch from
-    # pinned host memory and reads the clock's squared loss back.
+    # End to end through the public API: every clock's minibatch comes from
+    # pinned host memory (the copy of clock c+1 overlaps clock c) and every
+    # clock's squared loss goes back to the host.
     t.table_init(x0)
-    host_mb = [t.mf_export_minibatch(b) for b in range(w.F)]
+    need = sorted({(c - 1) % w.F for c in range(W + 1, W + K + 1)})
+    host_mb = {b: t.mf_export_minibatch(b) for b in need}
+    copy_stream = torch.cuda.Stream(dev)
     loss_d = torch.zeros(K, dtype=torch.float64, device=dev)
     loss_h = torch.empty(K, dtype=torch.float64, pin_memory=True)
     for _ in range(W):
         t.mf_sgd_clock(w.eta, w.lam, w.cap)
-    h2d = d2h = 0
+    b0 = (W + 1 - 1) % w.F
+    t.mf_stage_minibatch(b0, *host_mb[b0], stream=stream)  # sizes the staging buffer, outside the timing
     torch.cuda.synchronize(dev)
+    t.poll()
     _barrier(world)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     wall0 = time.time()
-    e0.record(stream)
-    with torch.cuda.stream(stream):
-        for k in range(K):
-            c = W + 1 + k
-            b = (c - 1) % w.F
-            u, j, D, uoff = host_mb[b]
-            t.mf_stage_minibatch(b, u, j, D, uoff)
-            h2d += 4 * (u.numel() + j.numel() + D.numel() + uoff.numel())
-            t.mf_sgd_clock(w.eta, w.lam, w.cap, sq_loss=loss_d[k:k + 1])
-            loss_h[k:k + 1].copy_(loss_d[k:k + 1], non_blocking=True)
-            d2h += 8
+    e0, h2d, d2h = _stage_overlapped(t, w, host_mb, W, K, stream, copy_stream, loss_d, loss_h)
+    e1 = torch.cuda.Event(enable_timing=True)
     e1.record(stream)
     torch.cuda.synchronize(dev)
     wall = time.time() - wall0
@@ -322,27 +382,17 @@ def run_gpu(args, w):
     e2e_ms = _max_over_ranks(world, e2e_ms)
     e2e_value = total_ratings / (e2e_ms / 1e3)
     t.poll()
+    del host_mb
 
     kern_avg_s = statistics.mean(kern_ms) / 1e3
     floor_avg = statistics.mean(floors)
     peak, peak_kind = _peaks()
     achieved = floor_avg / kern_avg_s / 1e9
-    kernel = "sgd_users32_kernel" if 64 < w.K <= 128 else "sgd_users_kernel"
+    kernel = _sgd_kernel_name(w.K)
     n_avg = ratings / K
-    B_model = 12 + 16 * w.K + 8 * w.K * (w.n_users + w.n_items) / n_avg
     out = {
-        "metric": METRIC,
         "value": value,
-        "unit": UNIT,
-        "n_gpus": world,
-        "steps": K,
-        "warmup": W,
         "ms_per_step": ms_max / K,
-        "higher_is_better": True,
-        "scaling": "weak",
-        "vs_baseline": None,
-        "dtype": "f32",
-        "data": "synthetic (seeded counter generator; Netflix-shaped, no real records)",
         "config": {
             "workload": f"{w.name}: {w.n_users}x{w.n_items}, {w.n_obs} entries, rank {w.K}, P={w.P}, "
                         f"F={w.F}, {w.model.upper()} s={w.s}"
@@ -355,36 +405,96 @@ def run_gpu(args, w):
         },
         "roofline": {
             "bound": "hbm",
-            "kernel": kernel + " (+ sgd_chunks_kernel / heavy_merge_kernel when some user is heavy)",
+            "kernel": kernel,
             "achieved": achieved,
             "peak": peak,
             "peak_kind": peak_kind,
             "unit": "GB/s",
             "frac": achieved / peak,
-            "traffic": _profiled_traffic(kernel, w.name),
+            "traffic": _profiled_traffic(kernel.split(" ")[0], w.name),
             "algorithmic_bytes_per_launch": floor_avg,
             "kernel_ms": statistics.mean(kern_ms),
-            "modelled_bytes_per_rating": B_model,
-            "modelled_GBps": n_avg * B_model / kern_avg_s / 1e9,
+            # compulsory bytes per rating of the SGD launch (the figure `achieved` uses)
+            "modelled_bytes_per_rating": floor_avg / n_avg,
+            # an upper bound that ignores every reuse in L2: 12 + 16K + 8K(N+M)/n
+            "no_reuse_bytes_per_rating": 12 + 16 * w.K + 8 * w.K * (w.n_users + w.n_items) / n_avg,
         },
-        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d // K, "d2h_bytes_per_step": d2h // K},
-        # per clock: the SGD kernel and the item merge (which also computes the
-        # next schedule), plus the chunk and heavy-merge kernels on minibatches
-        # with heavy users, plus the read model's own kernels
-        "gpu_launches": int(sum(2 + 2 * model.heavy[(c - 1) % w.F] + _model_launches(w, c)
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d // K, "d2h_bytes_per_step": d2h // K,
+                "copies": "minibatch of clock c+1 staged on a second stream while clock c runs"},
+        # per clock: the SGD kernels and the item merge (which also computes the
+        # next schedule), plus the read model's own kernels
+        "gpu_launches": int(sum(_sgd_launches(w.K, heavy[(c - 1) % w.F]) + _model_launches(w, c)
                                 for c in range(W + 1, W + K + 1))),
         "clocks": clocks,
         "objective": {"clock": c_final, "sq_loss": sq, "penalised": pen},
         # Fig. 1 (left) quantity: clock differential v_p(c) - c of every read in
         # the timed clocks (-1 = freshest version; BSP always gives -1).
         "clock_differential": {str(-1 - k): float(stale[k] / stale.sum()) for k in range(w.s + 1)},
-        "setup_s": {"generate": gen_s},
+        "setup_s": {"generate": gen_s, "load": load_s},
     }
+    t.close()
+    del t, x0
+    torch.cuda.empty_cache()
+    return out, data, (wp, mb)
+
+
+def _sgd_kernel_name(K):
+    """The SGD launches of one clock that the profile events bracket."""
+    if 32 < K <= 64:
+        return "sgd_work16_kernel (+ user_copy_kernel, and heavy_merge_kernel when some user is heavy)"
+    if 64 < K <= 128:
+        return "sgd_users32_kernel (+ sgd_chunks_kernel / heavy_merge_kernel when some user is heavy)"
+    return "sgd_users_kernel (+ sgd_chunks_kernel / heavy_merge_kernel when some user is heavy)"
+
+
+def _sgd_launches(K, heavy: bool) -> int:
+    """Kernels of one clock's SGD phase plus the item merge (which also
+    computes the next schedule)."""
+    if 32 < K <= 64:  # forward copy, work list, heavy merge
+        return 2 + int(heavy) + 1
+    return 1 + 2 * int(heavy) + 1
+
+
+def run_gpu(args, w):
+    import torch
+
+    from gen import workload
+
+    world, rank, local = _dist()
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    res, data, part = measure(args, w, dev, world, rank, local)
+    out = {
+        "metric": METRIC,
+        "value": res.pop("value"),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": res.pop("ms_per_step"),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic (seeded counter generator; Netflix-shaped, no real records)",
+    }
+    out.update(res)
+    extra = [x for x in args.extra.split(",") if x and x != "none" and x != w.name]
+    if extra:
+        out["extra_workloads"] = {}
+        for name in extra:
+            r, _, _ = measure(args, workload(name), dev, world, rank, local)
+            out["extra_workloads"][name] = r
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(w, data, (wp, mb), clocks=args.cpu_clocks)
+        out["cpu_baseline"] = cpu_baseline(w, data, part, clocks=args.cpu_clocks)
     if rank == 0:
         print(json.dumps(out), flush=True)
-    t.close()
     if world > 1:
         import torch.distributed as dist
 
@@ -462,10 +572,12 @@ def run_reference(args, w):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="esspt", choices=["esspt", "reference"])
-    ap.add_argument("--workload", default="mid")
+    ap.add_argument("--workload", default="large")
+    ap.add_argument("--extra", default="mid", help="comma-separated workloads also measured (reported under "
+                    "extra_workloads), or none")
     ap.add_argument("--cpu-clocks", type=int, default=2)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()

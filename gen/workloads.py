@@ -11,6 +11,8 @@
 * mid_row: the mid data under row-granular SSP (per-row cached versions), s=3.
 * large: 10M x 1M, 2B entries, Zipf(1.1) users and items, rank-64 model,
          128 workers, 1/50 per clock, SSP s=4, 20 clocks.
+* large_s: large's distributions at a fifth of its rows and per-clock entries
+         (2M x 200k, 80M entries, 1/10 per clock): the small profiling case.
 * sweep: the mid data with s in {0,1,2,4,8} x P in {1,8,64,512} x {SSP, ESSP},
          20 clocks each.
 """
@@ -65,12 +67,17 @@ class Workload:
             **self.data,
         )
 
+    def workers(self):
+        """user -> worker, int32[N]."""
+        return shard_users(self.n_users, self.P, self.data_seed + 1)
+
+    def minibatches(self):
+        """entry -> minibatch, uint8[n_obs]."""
+        return minibatch_labels(self.n_obs, self.F, self.data_seed + 2)
+
     def partition(self):
         """(user -> worker int32[N], entry -> minibatch uint8[n_obs])."""
-        return (
-            shard_users(self.n_users, self.P, self.data_seed + 1),
-            minibatch_labels(self.n_obs, self.F, self.data_seed + 2),
-        )
+        return self.workers(), self.minibatches()
 
     @property
     def ratings_per_clock(self) -> float:
@@ -114,6 +121,15 @@ WORKLOADS = {
     ),
     "large": Workload(
         "large", 10_000_000, 1_000_000, 2_000_000_000, K=64, P=128, F=50, s=4,
+        model="ssp", clocks=20, eta=0.005, lam=0.05, cap=20,
+        data=dict(user_dist="zipf", user_a=1.1, item_dist="zipf", item_a=1.1,
+                  truth_rank=32, truth_var=32 ** -0.5, noise_var=0.5),
+    ),
+    # The large workload's distributions at a fifth of its rows and entries
+    # per clock (2M x 200k, 8M entries per clock): the small case for ncu
+    # counter captures of the K=64 kernels, a few GB on the device.
+    "large_s": Workload(
+        "large_s", 2_000_000, 200_000, 80_000_000, K=64, P=128, F=10, s=4,
         model="ssp", clocks=20, eta=0.005, lam=0.05, cap=20,
         data=dict(user_dist="zipf", user_a=1.1, item_dist="zipf", item_a=1.1,
                   truth_rank=32, truth_var=32 ** -0.5, noise_var=0.5),

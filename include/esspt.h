@@ -250,12 +250,33 @@ esspt_status esspt_mf_minibatch_size(esspt_ctx* ctx, int32_t b, int64_t* n_b);
 esspt_status esspt_mf_export_minibatch(esspt_ctx* ctx, int32_t b, int32_t* h_u, int32_t* h_j, float* h_D,
                                        int32_t* h_uoff);
 
+/* Bytes of the device staging buffer esspt_mf_stage_minibatch() needs: the
+ * user and item ids of the largest minibatch plus one set of user offsets.
+ * 0 before esspt_mf_load(). */
+size_t esspt_mf_stage_bytes(const esspt_ctx* ctx);
+
 /* Copy minibatch b from host memory (the arrays esspt_mf_export_minibatch()
- * produced, possibly with new values h_D) into the device layout,
- * asynchronously on the stream (pinned host memory gives a true async copy).
- * The host arrays must stay valid until the stream reaches the copy. */
+ * produced, possibly with new values h_D) to the device, asynchronously on
+ * `stream` (cudaStream_t; NULL = the context's stream; pinned host memory
+ * gives a true async copy).  Together with esspt_mf_export_minibatch() this
+ * keeps the observed entries resident on the host, as each worker of
+ * Sec. 3.1 stores its own partition of D_obs.
+ *   h_D    replaces the values of minibatch b;
+ *   h_u, h_j, h_uoff  must be the loaded structure of minibatch b: they are
+ *          copied into `d_stage` (device, 256-byte aligned, caller-owned,
+ *          esspt_mf_stage_bytes() long) and compared on the device with the
+ *          loaded layout; any difference is latched and reported by
+ *          esspt_poll() as ESSPT_EINVAL.  The clock kernels never read the
+ *          staged structure, so a changed one cannot make them read outside
+ *          the table; only the new values take effect.
+ * The caller orders the call after the last clock that read minibatch b and
+ * before the next clock that reads it (e.g. with events when `stream` is not
+ * the context's stream).  Calls that overlap on the GPU must use different
+ * staging buffers.  The host arrays must stay valid until the stream reaches
+ * the copy.  ESSPT_ENOSPC if `stage_bytes` is short. */
 esspt_status esspt_mf_stage_minibatch(esspt_ctx* ctx, int32_t b, const int32_t* h_u, const int32_t* h_j,
-                                      const float* h_D, const int32_t* h_uoff);
+                                      const float* h_D, const int32_t* h_uoff, void* d_stage, size_t stage_bytes,
+                                      void* stream);
 
 /* Profiling hook: when `before` and `after` (cudaEvent_t) are non-NULL,
  * every following esspt_mf_sgd_clock() records `before` on the stream just

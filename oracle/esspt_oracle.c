@@ -90,6 +90,20 @@ static int orc_holds(const orc_state* st, int32_t version) {
   return version > st->version - st->nslots;
 }
 
+/* P(delay >= k) = (1-p)^k for a delay counted in failures before the first
+ * success; as a 32-bit threshold, floor((1-p)^k 2^32).  *q holds (1-p)^(k-1)
+ * on entry and (1-p)^k on return. */
+static uint32_t orc_threshold_next(double* q, double fail) {
+  *q *= fail;
+  return (uint32_t)floor(*q * 4294967296.0);
+}
+
+int orc_essp_thresholds(const orc_config* cfg, uint32_t* thr) {
+  double q = 1.0;
+  for (int32_t k = 1; k <= cfg->essp_max_delay; ++k) thr[k - 1] = orc_threshold_next(&q, 1.0 - cfg->essp_p);
+  return cfg->essp_max_delay;
+}
+
 int orc_schedule_rule(const orc_config* cfg, int32_t c, const int32_t* v_prev, int32_t* v_out) {
   int32_t lo = c - 1 - cfg->s;
   if (lo < 0) lo = 0;
@@ -107,13 +121,10 @@ int orc_schedule_rule(const orc_config* cfg, int32_t c, const int32_t* v_prev, i
        * delay >= k  iff  u < floor((1-essp_p)^k * 2^32). */
       int32_t dmax = cfg->essp_max_delay < cfg->s ? cfg->essp_max_delay : cfg->s;
       uint32_t u = (uint32_t)(orc_ctr_u64(cfg->seed, ORC_STREAM_DELAY, ((uint64_t)(uint32_t)c << 32) | (uint32_t)p) >> 32);
-      double q = 1.0, fail = 1.0 - cfg->essp_p;
+      double q = 1.0;
       int32_t delay = 0;
-      for (int32_t k = 1; k <= dmax; ++k) {
-        q *= fail;
-        uint32_t thr = (uint32_t)floor(q * 4294967296.0);
-        if (u < thr) delay = k;
-      }
+      for (int32_t k = 1; k <= dmax; ++k)
+        if (u < orc_threshold_next(&q, 1.0 - cfg->essp_p)) delay = k;
       v = c - 1 - delay;
       if (v_prev != NULL && v_prev[p] > v) v = v_prev[p];
       if (v < 0) v = 0;

@@ -99,6 +99,11 @@ int orc_table(const orc_state* st, int32_t version, double* out);
  * sq = sum e^2 (Sec. 5 squared loss), pen = sum [e^2 + lambda(|L_i|^2+|R_j|^2)]. */
 int orc_objective(const orc_state* st, int32_t version, double* sq, double* pen);
 
+/* ORC_ESSP_EAGER delay thresholds: thr[k-1] = floor((1-essp_p)^k 2^32) for
+ * k = 1..essp_max_delay (a delay is >= k iff the draw's top 32 bits are below
+ * thr[k-1]).  Returns essp_max_delay. */
+int orc_essp_thresholds(const orc_config* cfg, uint32_t* thr);
+
 /* Squared loss of the last clock: sum of e^2 over the entries of its
  * minibatch, each e taken where its update was computed (at the worker's
  * read version; in the sequential variant, at the worker's view just before

@@ -83,6 +83,8 @@ def _load():
         lib.orc_ctr_u64.restype = ctypes.c_uint64
         lib.orc_vap_norms.argtypes = [P, P, P]
         lib.orc_vap_norms.restype = ctypes.c_int
+        lib.orc_essp_thresholds.argtypes = [P, P]
+        lib.orc_essp_thresholds.restype = ctypes.c_int
         lib.orc_clock_loss.argtypes = [P, P]
         lib.orc_clock_loss.restype = ctypes.c_int
         lib.orc_row_version.argtypes = [P, ctypes.c_int32, ctypes.c_int64, P]
@@ -243,6 +245,14 @@ def schedule_rule(cfg: OracleConfig, c: int, v_prev=None):
     cc = cfg._c()
     rc = lib.orc_schedule_rule(ctypes.byref(cc), c, _ptr(prev), _ptr(out))
     return None if rc != 0 else out
+
+
+def essp_thresholds(cfg: OracleConfig) -> list:
+    """The ESSP delay thresholds floor((1-p)^k 2^32), k = 1..essp_max_delay."""
+    out = np.zeros(max(1, cfg.essp_max_delay), dtype=np.uint32)
+    cc = cfg._c()
+    n = _load().orc_essp_thresholds(ctypes.byref(cc), _ptr(out))
+    return [int(x) for x in out[:n]]
 
 
 def ctr_u64(seed: int, stream: int, index: int) -> int:

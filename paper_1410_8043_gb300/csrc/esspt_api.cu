@@ -38,6 +38,10 @@ struct esspt_ctx {
   int4 *chunk = nullptr, *heavy = nullptr;
   std::vector<int64_t> mb_base, chunk_base, heavy_base;
   cudaEvent_t ev_before = nullptr, ev_after = nullptr;
+  // Work-list path: the forward copy of idle users runs on a second stream
+  // beside the work kernel (created on first use, on the context's device).
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 };
 
 namespace {
@@ -198,7 +202,7 @@ struct MfCarve {
 // zero-initialised delta replicas dR (items) and dL (heavy users).
 MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int32_t K, bool row_mode) {
   MfCarve k{};
-  k.max_chunks = layout_max_chunks(n_obs, F);
+  k.max_chunks = layout_max_chunks(n_obs, F, n_users, uses_work16(K));
   k.max_heavy = layout_max_heavy(n_obs, F);
   k.dR_rows = layout_max_item_reps(n_obs, n_items);
   k.dL_rows = n_users + layout_max_user_reps(n_obs);
@@ -233,8 +237,14 @@ MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int
 }
 
 bool mf_sizes_ok(const esspt_ctx* c, int64_t n_obs, int64_t n_users, int32_t F) {
-  return c && n_obs >= 0 && n_obs < (int64_t)INT32_MAX && n_users > 0 && n_users < c->n_rows && F >= 1 &&
-         F <= 255 && (int64_t)F * n_users < (int64_t)INT32_MAX;
+  if (!(c && n_obs >= 0 && n_obs < (int64_t)INT32_MAX && n_users > 0 && n_users < c->n_rows && F >= 1 && F <= 255 &&
+        (int64_t)F * n_users < (int64_t)INT32_MAX))
+    return false;
+  // The SGD kernels offset item rows and item replica rows by 32-bit float4
+  // products (item * K/4, replica row * row stride).
+  const int64_t n_items = c->n_rows - n_users;
+  return n_items * (c->K / 4) < (int64_t)INT32_MAX &&
+         layout_max_item_reps(n_obs, n_items) * dR_stride4(c->K) < (int64_t)INT32_MAX;
 }
 
 }  // namespace
@@ -324,6 +334,12 @@ esspt_status esspt_create(const esspt_config* cfg, void* d_workspace, size_t byt
 esspt_status esspt_destroy(esspt_ctx* c) {
   if (!c) return ESSPT_OK;
   cudaError_t e = cudaStreamSynchronize(c->st);
+  if (c->side) {
+    cudaStreamSynchronize(c->side);
+    cudaStreamDestroy(c->side);
+  }
+  if (c->ev_fork) cudaEventDestroy(c->ev_fork);
+  if (c->ev_join) cudaEventDestroy(c->ev_join);
   delete c;
   return e == cudaSuccess ? ESSPT_OK : ESSPT_ECUDA;
 }
@@ -484,6 +500,7 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   b.heavy = reinterpret_cast<int4*>(w + k.heavy);
   b.heavy_base = reinterpret_cast<int64_t*>(w + k.heavy_base);
   b.max_chunks = k.max_chunks;
+  b.light_items = uses_work16(c->K);
   b.max_heavy = k.max_heavy;
   b.scratch = d_scratch;
   b.scratch_bytes = scratch_bytes;
@@ -603,15 +620,36 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   const int64_t nch = c->chunk_base[b + 1] - c->chunk_base[b];
   const int64_t nhv = c->heavy_base[b + 1] - c->heavy_base[b];
   if (c->ev_before) ESSPT_CUDA(c, cudaEventRecord(c->ev_before, c->st));
-  if (nch > 0) {
-    ChunkArgs ch{};
-    ch.a = a;
-    ch.chunk = c->chunk + c->chunk_base[b];
-    ch.n_chunks = nch;
-    ch.dL = c->dL;
-    ESSPT_CUDA(c, launch_sgd_chunks(ch, c->st));
+  ChunkArgs ch{};
+  ch.a = a;
+  ch.chunk = c->chunk + c->chunk_base[b];
+  ch.n_chunks = nch;
+  ch.dL = c->dL;
+  if (uses_work16(c->K)) {
+    // Work-list path: users without entries are copied forward; every other
+    // user (and every chunk of a heavy user) is one item of the work kernel.
+    // The copy is HBM streaming and the work kernel mostly L2 traffic, so the
+    // copy runs on a second stream beside it.
+    if (kForkCopy) {
+      if (!c->side) {
+        ESSPT_CUDA(c, cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking));
+        ESSPT_CUDA(c, cudaEventCreateWithFlags(&c->ev_fork, cudaEventDisableTiming));
+        ESSPT_CUDA(c, cudaEventCreateWithFlags(&c->ev_join, cudaEventDisableTiming));
+      }
+      ESSPT_CUDA(c, cudaEventRecord(c->ev_fork, c->st));
+      ESSPT_CUDA(c, cudaStreamWaitEvent(c->side, c->ev_fork, 0));
+      ESSPT_CUDA(c, launch_user_copy(a, c->side));
+      ESSPT_CUDA(c, cudaEventRecord(c->ev_join, c->side));
+      ESSPT_CUDA(c, launch_sgd_work16(ch, c->st));
+      ESSPT_CUDA(c, cudaStreamWaitEvent(c->st, c->ev_join, 0));
+    } else {
+      ESSPT_CUDA(c, launch_user_copy(a, c->st));
+      ESSPT_CUDA(c, launch_sgd_work16(ch, c->st));
+    }
+  } else {
+    if (nch > 0) ESSPT_CUDA(c, launch_sgd_chunks(ch, c->st));
+    ESSPT_CUDA(c, launch_sgd_users(a, c->st));
   }
-  ESSPT_CUDA(c, launch_sgd_users(a, c->st));
   if (nhv > 0) {
     HeavyMergeArgs h{};
     h.ring = c->ring;
@@ -739,18 +777,37 @@ esspt_status esspt_mf_export_minibatch(esspt_ctx* c, int32_t b, int32_t* h_u, in
   return ESSPT_OK;
 }
 
+size_t esspt_mf_stage_bytes(const esspt_ctx* c) {
+  if (!c || !c->mf) return 0;
+  int64_t mx = 0;
+  for (int32_t b = 0; b < c->F; ++b) mx = std::max(mx, c->mb_base[b + 1] - c->mb_base[b]);
+  return 2 * align256(sizeof(int32_t) * (size_t)mx) + align256(sizeof(int32_t) * (size_t)(c->n_users + 1));
+}
+
 esspt_status esspt_mf_stage_minibatch(esspt_ctx* c, int32_t b, const int32_t* h_u, const int32_t* h_j,
-                                      const float* h_D, const int32_t* h_uoff) {
+                                      const float* h_D, const int32_t* h_uoff, void* d_stage, size_t stage_bytes,
+                                      void* stream) {
   int64_t n = 0;
   esspt_status s = esspt_mf_minibatch_size(c, b, &n);
   if (s != ESSPT_OK) return s;
   if (!h_u || !h_j || !h_D || !h_uoff) return fail(c, ESSPT_EINVAL, "null host buffer");
+  if (!d_stage || (reinterpret_cast<uintptr_t>(d_stage) & 255u)) return fail(c, ESSPT_EINVAL, "stage must be 256-byte aligned");
+  if (stage_bytes < esspt_mf_stage_bytes(c)) return fail(c, ESSPT_ENOSPC, "staging buffer too small");
+  cudaStream_t st = stream ? static_cast<cudaStream_t>(stream) : c->st;
   const int64_t base = c->mb_base[b];
-  ESSPT_CUDA(c, cudaMemcpyAsync(c->rec_u + base, h_u, sizeof(int32_t) * n, cudaMemcpyHostToDevice, c->st));
-  ESSPT_CUDA(c, cudaMemcpyAsync(c->rec_j + base, h_j, sizeof(int32_t) * n, cudaMemcpyHostToDevice, c->st));
-  ESSPT_CUDA(c, cudaMemcpyAsync(c->rec_D + base, h_D, sizeof(float) * n, cudaMemcpyHostToDevice, c->st));
-  ESSPT_CUDA(c, cudaMemcpyAsync(c->uoff + (int64_t)b * (c->n_users + 1), h_uoff, sizeof(int32_t) * (c->n_users + 1),
-                                cudaMemcpyHostToDevice, c->st));
+  // The values go straight into the layout; the structure only into the
+  // staging buffer, where it is compared with the loaded one.
+  char* w = static_cast<char*>(d_stage);
+  int32_t* su = reinterpret_cast<int32_t*>(w);
+  int32_t* sj = reinterpret_cast<int32_t*>(w + align256(sizeof(int32_t) * (size_t)n));
+  int32_t* suoff = reinterpret_cast<int32_t*>(w + 2 * align256(sizeof(int32_t) * (size_t)n));
+  int32_t* ruoff = c->uoff + (int64_t)b * (c->n_users + 1);
+  ESSPT_CUDA(c, cudaMemcpyAsync(c->rec_D + base, h_D, sizeof(float) * n, cudaMemcpyHostToDevice, st));
+  ESSPT_CUDA(c, cudaMemcpyAsync(su, h_u, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
+  ESSPT_CUDA(c, cudaMemcpyAsync(sj, h_j, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
+  ESSPT_CUDA(c, cudaMemcpyAsync(suoff, h_uoff, sizeof(int32_t) * (c->n_users + 1), cudaMemcpyHostToDevice, st));
+  ESSPT_CUDA(c, launch_stage_check(su, sj, suoff, c->rec_u + base, c->rec_j + base, ruoff, n, c->n_users + 1,
+                                   c->status, st));
   return ESSPT_OK;
 }
 

@@ -41,6 +41,21 @@ constexpr int32_t kUserRep = 64;
 #endif
 constexpr int32_t kMaxRep = ESSPT_MAX_REP;
 
+// Rows of 36..64 values (9..16 float4 slices) take the work-list path: every
+// user with 1..kHeavy entries in a minibatch is one work item beside the
+// chunks of the heavy users, processed by one kernel, and the users without
+// entries are copied forward by a streaming kernel.
+inline bool uses_work16(int32_t K) { return K > 32 && K <= 64; }
+// Run the forward copy of idle users on a second stream beside the work
+// kernel (each then takes part of every SM: kernels sized by kCopyBlocksPerSm
+// and kWorkBlocksPerSm).
+#ifndef ESSPT_FORK_COPY
+#define ESSPT_FORK_COPY 0
+#endif
+constexpr bool kForkCopy = ESSPT_FORK_COPY != 0;
+constexpr int kCopyBlocksPerSm = kForkCopy ? 1 : 8;
+constexpr int kWorkBlocksPerSm = kForkCopy ? 2 : 8;
+
 // Row stride (in float4) of the item delta replicas: K rounded up to a whole
 // number of 32-byte sectors, so that a row's reductions touch the fewest sectors.
 inline int32_t dR_stride4(int32_t K) { return ((K + 7) / 8) * 2; }
@@ -83,6 +98,8 @@ struct SgdArgs {
 };
 
 // Chunks of heavy users: x = user, y = begin, z = end (relative), w = replica row in dL.
+// On the work-list path a user with 1..kHeavy entries is one item with w = -1
+// (its row of version c is written directly).
 struct ChunkArgs {
   SgdArgs a;
   const int4* chunk;
@@ -169,6 +186,10 @@ struct SeqArgs {
 };
 cudaError_t launch_seq_clock(const SeqArgs& a, cudaStream_t st);
 cudaError_t launch_sgd_chunks(const ChunkArgs& a, cudaStream_t st);
+// Work-list path (uses_work16): the items of minibatch b (light users and
+// heavy-user chunks) and the forward copy of the users without entries.
+cudaError_t launch_sgd_work16(const ChunkArgs& a, cudaStream_t st);
+cudaError_t launch_user_copy(const SgdArgs& a, cudaStream_t st);
 cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st);
 cudaError_t launch_item_merge(const ItemMergeArgs& a, cudaStream_t st);
 cudaError_t launch_objective(const float* slot, int64_t n_users, int32_t K, const int32_t* rec_u,
@@ -198,6 +219,7 @@ struct LayoutBuild {
   int4* heavy;          // [max_heavy]
   int64_t* heavy_base;  // [F+1]
   int64_t max_chunks, max_heavy;
+  bool light_items;     // also list every user with 1..kHeavy entries (work-list path)
   // scratch
   void* scratch;
   size_t scratch_bytes;
@@ -205,12 +227,17 @@ struct LayoutBuild {
 };
 
 size_t layout_scratch_bytes(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F);
-int64_t layout_max_chunks(int64_t n_obs, int32_t F);
+int64_t layout_max_chunks(int64_t n_obs, int32_t F, int64_t n_users, bool light_items);
 int64_t layout_max_heavy(int64_t n_obs, int32_t F);
 int64_t layout_max_item_reps(int64_t n_obs, int64_t n_items);
 int64_t layout_max_user_reps(int64_t n_obs);
 cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st);
 cudaError_t launch_validate(const LayoutBuild& b, cudaStream_t st);
+// Staged minibatch check: su/sj (n entries) and suoff (n_off offsets) against
+// the resident ru/rj/ruoff; a difference latches kErrInput.
+cudaError_t launch_stage_check(const int32_t* su, const int32_t* sj, const int32_t* suoff, const int32_t* ru,
+                               const int32_t* rj, const int32_t* ruoff, int64_t n, int64_t n_off, uint32_t* status,
+                               cudaStream_t st);
 
 // Read-only view of a context's loaded MF entries and of table version
 // `version` (checked against the live window), for entry points defined in

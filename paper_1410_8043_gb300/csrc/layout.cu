@@ -80,7 +80,8 @@ __global__ void gather_kernel(const uint32_t* __restrict__ perm, int64_t n_obs, 
 // per (b, u): chunks, heavy flag and extra replica rows.
 __global__ void offsets_kernel(const int64_t* __restrict__ off, int64_t n_users, int32_t F, int32_t* __restrict__ uoff,
                                int64_t* __restrict__ mb_base, const int32_t* __restrict__ cnt,
-                               int32_t* __restrict__ nch, int32_t* __restrict__ hflag, int32_t* __restrict__ hextra) {
+                               int32_t* __restrict__ nch, int32_t* __restrict__ hflag, int32_t* __restrict__ hextra,
+                               bool light_items) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t total = (int64_t)F * (n_users + 1);
   for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < total; x += stride) {
@@ -91,7 +92,7 @@ __global__ void offsets_kernel(const int64_t* __restrict__ off, int64_t n_users,
     if (u < n_users) {
       const int32_t n = cnt[b * n_users + u];
       const int32_t c = n > kHeavy ? (n + kChunk - 1) / kChunk : 0;
-      nch[b * n_users + u] = c;
+      nch[b * n_users + u] = c + (light_items && n > 0 && c == 0 ? 1 : 0);
       hflag[b * n_users + u] = c > 0 ? 1 : 0;
       hextra[b * n_users + u] = c > 0 ? user_reps(c) - 1 : 0;
     }
@@ -115,6 +116,14 @@ __global__ void heavy_kernel(const int64_t* __restrict__ choff, const int32_t* _
     if (nc == 0) continue;
     const int64_t b = x / n_users, u = x % n_users;
     const int32_t beg = uoff[b * (n_users + 1) + u], end = uoff[b * (n_users + 1) + u + 1];
+    if (end - beg <= kHeavy) {  // a light user: one work item, written directly
+      if (choff[x] >= max_chunks) {
+        atomicOr(status, kErrInput);
+        continue;
+      }
+      chunk[choff[x]] = make_int4((int32_t)u, beg, end, -1);
+      continue;
+    }
     const int32_t reps = user_reps(nc);
     const int64_t extra0 = n_users + hext[x];
     // The bounds below hold by construction; the checks keep every store in range.
@@ -163,6 +172,21 @@ __global__ void dst_kernel(const uint32_t* __restrict__ key, const int64_t* __re
     const int32_t r0 = item_rep[j], r1 = item_rep[j + 1];
     rec_dst[k] = r0 + (int32_t)(t & (int64_t)(r1 - r0 - 1));
   }
+}
+
+// A staged minibatch against the loaded one: every user id, item id and
+// user offset must be equal; any difference latches kErrInput.
+__global__ void stage_check_kernel(const int32_t* __restrict__ su, const int32_t* __restrict__ sj,
+                                   const int32_t* __restrict__ suoff, const int32_t* __restrict__ ru,
+                                   const int32_t* __restrict__ rj, const int32_t* __restrict__ ruoff, int64_t n,
+                                   int64_t n_off, uint32_t* status) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  bool bad = false;
+  for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < n; k += stride)
+    bad |= su[k] != ru[k] || sj[k] != rj[k];
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < n_off; u += stride)
+    bad |= suoff[u] != ruoff[u];
+  if (__any_sync(0xffffffffu, bad) && (threadIdx.x & 31) == 0) atomicOr(status, kErrInput);
 }
 
 int blocks_for(int64_t n) {
@@ -225,7 +249,10 @@ size_t layout_scratch_bytes(int64_t n_obs, int64_t n_users, int64_t n_items, int
 }
 
 // A heavy segment has n > kHeavy >= kChunk entries and ceil(n/kChunk) < 2n/kChunk chunks.
-int64_t layout_max_chunks(int64_t n_obs, int32_t F) { return 2 * n_obs / kChunk + F + 1; }
+// On the work-list path every user with entries in a minibatch adds one more item.
+int64_t layout_max_chunks(int64_t n_obs, int32_t F, int64_t n_users, bool light_items) {
+  return 2 * n_obs / kChunk + F + 1 + (light_items ? std::min(n_obs, (int64_t)F * n_users) : 0);
+}
 
 int64_t layout_max_heavy(int64_t n_obs, int32_t F) { return n_obs / (kHeavy + 1) + F + 1; }
 
@@ -273,7 +300,8 @@ cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st) {
   size_t tb = p.cub_bytes;
   if ((e = cub::DeviceScan::ExclusiveSum(cub_tmp, tb, cnt, off, (int)(keys + 1), st)) != cudaSuccess) return e;
   offsets_kernel<<<blocks_for((int64_t)b.F * (b.n_users + 1)), 256, 0, st>>>(off, b.n_users, b.F, b.uoff, b.mb_base,
-                                                                            cnt, nch, hflag, hextra);
+                                                                            cnt, nch, hflag, hextra,
+                                                                            b.light_items);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   tb = p.cub_bytes;
   if ((e = cub::DeviceScan::ExclusiveSum(cub_tmp, tb, nch, choff, (int)(keys + 1), st)) != cudaSuccess) return e;
@@ -293,6 +321,13 @@ cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st) {
   if (b.n_obs == 0) return cudaSuccess;
   dst_kernel<<<blocks_for(b.n_obs), 256, 0, st>>>(key_out, b.mb_base, b.rec_j, b.item_rep, b.n_obs, b.n_users,
                                                   b.rec_dst);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_stage_check(const int32_t* su, const int32_t* sj, const int32_t* suoff, const int32_t* ru,
+                               const int32_t* rj, const int32_t* ruoff, int64_t n, int64_t n_off, uint32_t* status,
+                               cudaStream_t st) {
+  stage_check_kernel<<<blocks_for(std::max(n, n_off)), 256, 0, st>>>(su, sj, suoff, ru, rj, ruoff, n, n_off, status);
   return cudaGetLastError();
 }
 

@@ -524,6 +524,268 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
   flush_loss(a.sq_loss, loss, lane);
 }
 
+// Rows of 36..64 values (9..16 float4 slices) on the work-list path.
+//
+// sgd_work16_kernel: one warp per work item of minibatch b, either a user
+// with 1..kHeavy entries (written once: L^c = L^base + eta s sum_k(e_k R_j -
+// lambda L_i)) or a 64-entry chunk of a heavy user (its unscaled partial sum
+// goes into the chunk's replica row of dL, merged by heavy_merge_kernel).
+// Both halves of the warp hold the item's row L_i (lane l owns slice l mod
+// 16); a step takes 8 entries, half h the entries 2m + h (m = 0..3), so each
+// gather instruction brings two item rows.  A transposing butterfly over the
+// 16 lanes of a half (4 shuffles) leaves entry 2m + h's dot product on lanes
+// 4m .. 4m+3 of half h.  The item's rows at the read and base versions are
+// staged in shared memory one item ahead by cp.async, and each warp walks one
+// contiguous range of items, balanced by entries plus kItemCost per item.
+#ifndef ESSPT_WORK16_MINB
+#define ESSPT_WORK16_MINB 3
+#endif
+#ifndef ESSPT_W16_ITEMCOST
+#define ESSPT_W16_ITEMCOST 6
+#endif
+constexpr int32_t kItemCost = ESSPT_W16_ITEMCOST;
+constexpr int kW16Unit = 16;
+
+__global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(ChunkArgs c) {
+  const SgdArgs& a = c.a;
+  __shared__ __align__(16) float4 stage[8][2][2][16];  // [warp][buffer][read row, base row][slice]
+  const int lane = threadIdx.x & 31;
+  const int wib = threadIdx.x >> 5;
+  const int h = lane >> 4;      // half: entries 2m + h of a step
+  const int r = lane & 15;      // slice of the row this lane owns
+  const int32_t K4 = a.K >> 2;
+  const bool on = r < K4;
+  const int64_t slot4 = a.n_rows * K4;
+  float4* ring4 = reinterpret_cast<float4*>(a.ring);
+  float4* outq = ring4 + (int64_t)a.slot_out * slot4;
+  const float4* base4 = ring4 + (int64_t)a.slot_base * slot4;
+  float4* dRq = reinterpret_cast<float4*>(a.dR) + (on ? r : 0);
+  float4* dL4 = reinterpret_cast<float4*>(c.dL);
+  const int32_t n_items = (int32_t)c.n_chunks;
+  const uint64_t pol = policy_evict_first();
+  float loss = 0.f;
+
+  // Item x starts at entry chunk[x].y; the entries of consecutive items are
+  // contiguous, so the cost of items [0, x) is chunk[x].y + kItemCost x.
+  auto item_beg = [&](int32_t x) -> int64_t { return x < n_items ? (int64_t)__ldg(&c.chunk[x].y) : (int64_t)a.n_b; };
+  int32_t ia, ib;
+  {
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int half = lane >> 4, hl = lane & 15;
+    const int64_t total = (int64_t)a.n_b + (int64_t)kItemCost * n_items;
+    const int64_t target = total * (w + half) / nw;
+    int32_t lo = 0, hi = n_items;
+    while (__any_sync(0xffffffffu, lo < hi)) {
+      const int32_t step = (hi - lo + 15) / 16;
+      const int32_t x = (int32_t)min((int64_t)lo + (int64_t)hl * step, (int64_t)hi);
+      const bool ge = lo < hi && item_beg(x) + (int64_t)kItemCost * x >= target;
+      const unsigned bits = (__ballot_sync(0xffffffffu, ge) >> (16 * half)) & 0xffffu;
+      if (lo < hi) {
+        if (bits == 0u) {
+          lo = (int32_t)min((int64_t)lo + (int64_t)15 * step, (int64_t)hi) + 1;
+        } else {
+          const int f = __ffs(bits) - 1;
+          const int32_t xf = (int32_t)min((int64_t)lo + (int64_t)f * step, (int64_t)hi);
+          if (f == 0) {
+            hi = lo;
+          } else {
+            lo = (int32_t)min((int64_t)lo + (int64_t)(f - 1) * step, (int64_t)hi) + 1;
+            hi = xf;
+          }
+        }
+      }
+    }
+    ia = __shfl_sync(0xffffffffu, lo, 0);
+    ib = __shfl_sync(0xffffffffu, lo, 16);
+  }
+  if (ia >= ib) {
+    flush_loss(a.sq_loss, 0.f, lane);
+    return;
+  }
+
+  // Item metadata: the current unit in lanes [0, 16), the next in [16, 32).
+  int4 m_it = make_int4(0, 0, 0, 0);
+  int32_t m_vs = 0;
+  auto load_meta = [&](int64_t first, int lo) {
+    if (lane >= lo && lane < lo + kW16Unit) {
+      const int64_t x = first + (lane - lo);
+      m_it = make_int4(0, 0, 0, 0);
+      m_vs = 0;
+      if (x < ib) {
+        m_it = __ldg(c.chunk + x);
+        m_vs = user_slot(a, m_it.x);
+      }
+    }
+  };
+  // Stage item ml's rows: lanes [0, 16) its read-version row, lanes [16, 32)
+  // its base row (only a light user whose read version is not the base).
+  auto stage_item = [&](int ml, int bb) {
+    const int32_t u = __shfl_sync(0xffffffffu, m_it.x, ml);
+    const int32_t dst = __shfl_sync(0xffffffffu, m_it.w, ml);
+    const int32_t vs = __shfl_sync(0xffffffffu, m_vs, ml);
+    const bool same = vs == a.slot_base;
+    const int64_t row = (int64_t)u * K4 + (on ? r : 0);
+    if (h == 0)
+      cp_async16_hint(&stage[wib][bb][0][r], ring4 + (int64_t)vs * slot4 + row, on, pol);
+    else
+      cp_async16_hint(&stage[wib][bb][1][r], base4 + row, on && dst < 0 && !same, pol);
+    cp_async_commit();
+  };
+
+  load_meta(ia, 0);
+  load_meta((int64_t)ia + kW16Unit, kW16Unit);
+  Window<32> win;
+  stage_item(0, 0);
+  win.reload(a, __shfl_sync(0xffffffffu, m_it.y, 0), lane);
+  int bb = 0;
+  for (int64_t x0 = ia; x0 < ib; x0 += kW16Unit) {
+    const int32_t nloc = (int32_t)min((int64_t)kW16Unit, (int64_t)ib - x0);
+    for (int32_t t = 0; t < nloc; ++t, bb ^= 1) {
+      cp_async_wait_all();
+      __syncwarp();
+      if (t + 1 < nloc) {
+        stage_item(t + 1, bb ^ 1);
+      } else if (x0 + kW16Unit < ib) {
+        stage_item(kW16Unit, bb ^ 1);
+      }
+      const int32_t u = __shfl_sync(0xffffffffu, m_it.x, t);
+      const int32_t beg = __shfl_sync(0xffffffffu, m_it.y, t);
+      const int32_t end = __shfl_sync(0xffffffffu, m_it.z, t);
+      const int32_t dst = __shfl_sync(0xffffffffu, m_it.w, t);
+      const int32_t vs = __shfl_sync(0xffffffffu, m_vs, t);
+      const float4 Lv = stage[wib][bb][0][r];
+      // Lanes past the row end read slice 0 of the item rows; their staged L is
+      // zero, so they add nothing to the dot products.
+      const float4* Rq =
+          (a.row_mode ? ring4 : ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4) + (on ? r : 0);
+      float4 gL = f4_zero();
+      auto step = [&](auto full_tag, int32_t tt, int32_t cnt) {
+        constexpr bool kFull = decltype(full_tag)::value;
+        const int w0 = tt - win.W;
+        float4 R[4];
+        int32_t dsts[4];
+        float p[4];
+#pragma unroll
+        for (int m = 0; m < 4; ++m) {
+          const int k = 2 * m + h;
+          const int src = kFull ? w0 + k : min(w0 + k, 31);
+          const int32_t j = __shfl_sync(0xffffffffu, win.cj, src);
+          dsts[m] = __shfl_sync(0xffffffffu, win.cdst, src);
+          R[m] = (kFull || k < cnt) ? __ldg(Rq + j * K4) : f4_zero();
+          p[m] = dot4(Lv, R[m]);
+        }
+        // Transposing butterfly over the 16 lanes of a half: bit 3 of the
+        // lane keeps entries {0,1} or {2,3}, bit 2 one of the pair, bits 1
+        // and 0 sum; lanes 4m .. 4m+3 end with entry 2m + h's dot product.
+        const bool b3 = r & 8, b2 = r & 4;
+        float k0 = b3 ? p[2] : p[0], k1 = b3 ? p[3] : p[1];
+        k0 += __shfl_xor_sync(0xffffffffu, b3 ? p[0] : p[2], 8);
+        k1 += __shfl_xor_sync(0xffffffffu, b3 ? p[1] : p[3], 8);
+        float dot = b2 ? k1 : k0;
+        dot += __shfl_xor_sync(0xffffffffu, b2 ? k0 : k1, 4);
+        dot += __shfl_xor_sync(0xffffffffu, dot, 2);
+        dot += __shfl_xor_sync(0xffffffffu, dot, 1);
+        const int kq = 2 * (r >> 2) + h;  // the entry this lane's dot product belongs to
+        const float dq = __shfl_sync(0xffffffffu, win.cd, kFull ? w0 + kq : min(w0 + kq, 31));
+        const float eq = (kFull || kq < cnt) ? dq - dot : 0.f;
+        if ((r & 3) == 0) loss += eq * eq;
+#pragma unroll
+        for (int m = 0; m < 4; ++m) {
+          const float e = __shfl_sync(0xffffffffu, eq, (lane & 16) + 4 * m);
+          const float4 rr = R[m];
+          gL.x += e * rr.x;
+          gL.y += e * rr.y;
+          gL.z += e * rr.z;
+          gL.w += e * rr.w;
+          red_add_v4_if(dRq + dsts[m] * a.dR_ld,
+                        make_float4(e * Lv.x - a.lambda * rr.x, e * Lv.y - a.lambda * rr.y,
+                                    e * Lv.z - a.lambda * rr.z, e * Lv.w - a.lambda * rr.w),
+                        on && (kFull || 2 * m + h < cnt));
+        }
+      };
+      for (int32_t tt = beg; tt < end;) {
+        win.cover(a, tt, lane);
+        const int32_t cnt = min(8, min(end - tt, win.W + 32 - tt));
+        if (cnt == 8) {
+          step(std::true_type{}, tt, cnt);
+        } else {
+          step(std::false_type{}, tt, cnt);
+        }
+        tt += cnt;
+      }
+      // both halves' sums, then the -lambda L_i term of every entry
+      gL.x += __shfl_xor_sync(0xffffffffu, gL.x, 16);
+      gL.y += __shfl_xor_sync(0xffffffffu, gL.y, 16);
+      gL.z += __shfl_xor_sync(0xffffffffu, gL.z, 16);
+      gL.w += __shfl_xor_sync(0xffffffffu, gL.w, 16);
+      const int32_t n = end - beg;
+      const float4 g = f4_axpy(-(float)n * a.lambda, Lv, gL);
+      if (dst >= 0) {  // a heavy user's chunk: unscaled partial sum into its replica row
+        if (h == 0 && on) red_add_v4(dL4 + (int64_t)dst * K4 + r, g);
+      } else {
+        const bool same = vs == a.slot_base;
+        const float4 lb = same ? Lv : stage[wib][bb][1][r];
+        float sc = a.eta;
+        if (a.cap > 0 && n > a.cap) sc = a.eta * capped_scale(a.cap, n);
+        st_stream_if(outq + (int64_t)u * K4 + r, f4_axpy(sc, g, lb), pol, h == 0 && on);
+      }
+    }
+    m_it.x = __shfl_down_sync(0xffffffffu, m_it.x, kW16Unit);
+    m_it.y = __shfl_down_sync(0xffffffffu, m_it.y, kW16Unit);
+    m_it.z = __shfl_down_sync(0xffffffffu, m_it.z, kW16Unit);
+    m_it.w = __shfl_down_sync(0xffffffffu, m_it.w, kW16Unit);
+    m_vs = __shfl_down_sync(0xffffffffu, m_vs, kW16Unit);
+    load_meta(x0 + 2 * kW16Unit, kW16Unit);
+    __syncwarp();
+  }
+  cp_async_wait_all();
+  flush_loss(a.sq_loss, loss, lane);
+}
+
+// Forward copy of the users with no entry in minibatch b (version c-1 row to
+// version c), on the work-list path.  One warp per 32 consecutive users: their
+// entry counts come from two coalesced offset loads, and the warp copies the
+// rows of the idle ones, all loads of a unit in flight before the stores.
+#ifndef ESSPT_COPY_BATCH
+#define ESSPT_COPY_BATCH 8
+#endif
+__global__ void __launch_bounds__(256, 4) user_copy_kernel(SgdArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int h = lane >> 4, r = lane & 15;
+  const int32_t K4 = a.K >> 2;
+  const bool on = r < K4;
+  const int64_t slot4 = a.n_rows * K4;
+  float4* ring4 = reinterpret_cast<float4*>(a.ring);
+  float4* outq = ring4 + (int64_t)a.slot_out * slot4;
+  const float4* base4 = ring4 + (int64_t)a.slot_base * slot4;
+  const uint64_t pol = policy_evict_first();
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t u0 = warp * 32; u0 < a.n_users; u0 += nwarps * 32) {
+    const int64_t u = u0 + lane;
+    bool idle = false;
+    if (u < a.n_users) idle = __ldg(a.uoff + u + 1) == __ldg(a.uoff + u);
+    const unsigned mask = __ballot_sync(0xffffffffu, idle);
+    if (mask == 0u) continue;
+    // rows 2q + h of the unit, q = 0..15, in batches
+    const int64_t first = (u0 + h) * K4 + (on ? r : 0);
+    const float4* src = base4 + first;
+    float4* dst = outq + first;
+    const unsigned mine = on ? (mask >> h) : 0u;  // bit q: row 2q + h is idle
+#pragma unroll 1
+    for (int q0 = 0; q0 < 16; q0 += ESSPT_COPY_BATCH) {
+      float4 v[ESSPT_COPY_BATCH];
+#pragma unroll
+      for (int q = 0; q < ESSPT_COPY_BATCH; ++q)
+        v[q] = ld_stream_if(src + (q0 + q) * 2 * K4, pol, (mine >> (2 * (q0 + q))) & 1u);
+#pragma unroll
+      for (int q = 0; q < ESSPT_COPY_BATCH; ++q)
+        st_stream_if(dst + (q0 + q) * 2 * K4, v[q], pol, (mine >> (2 * (q0 + q))) & 1u);
+    }
+  }
+}
+
 // Row-granular SSP (Sec. 4 client cache, a clock c_param per cached row):
 // thread x refreshes user x's row (if the user has entries) and entry x's
 // item row in the cache of the reading worker.  All threads that refresh one
@@ -735,6 +997,26 @@ cudaError_t launch_sgd_users(const SgdArgs& a, cudaStream_t st) {
 }
 cudaError_t launch_sgd_chunks(const ChunkArgs& c, cudaStream_t st) { return dispatch_k<ChunksF>(c.a.K, c, st); }
 
+// One resident wave of sgd_work16_kernel; its warps balance the items among
+// themselves.
+cudaError_t launch_sgd_work16(const ChunkArgs& c, cudaStream_t st) {
+  if (c.n_chunks <= 0) return cudaSuccess;
+  static int per_sm = 0;
+  if (per_sm == 0 &&
+      (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sgd_work16_kernel, 256, 0) != cudaSuccess ||
+       per_sm <= 0))
+    per_sm = 1;
+  sgd_work16_kernel<<<grid_for((c.n_chunks + kW16Unit - 1) / kW16Unit, 8, std::min(per_sm, kWorkBlocksPerSm)), 256,
+                      0, st>>>(c);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_user_copy(const SgdArgs& a, cudaStream_t st) {
+  if (a.n_users <= 0) return cudaSuccess;
+  user_copy_kernel<<<grid_for((a.n_users + 31) / 32, 8, kCopyBlocksPerSm), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_row_refresh(const RowRefreshArgs& a, cudaStream_t st) {
   const int64_t n = std::max<int64_t>(a.n_users, a.n_b);
   if (n <= 0) return cudaSuccess;
@@ -751,7 +1033,11 @@ cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st) {
 cudaError_t launch_item_merge(const ItemMergeArgs& a, cudaStream_t st) {
   const int64_t work = std::max<int64_t>((int64_t)a.n_items * (a.K >> 2), a.do_schedule ? a.sched.P : 0);
   if (work <= 0) return cudaSuccess;
-  item_merge_kernel<<<grid_for(work, 256, 16), 256, 0, st>>>(a);
+  // One thread per (item, slice): every thread's loads are independent, so
+  // the whole merge is one set of in-flight requests rather than a
+  // grid-stride chain of dependent ones.
+  const int64_t blocks = std::min<int64_t>((work + 255) / 256, (int64_t)1 << 30);
+  item_merge_kernel<<<(unsigned)blocks, 256, 0, st>>>(a);
   return cudaGetLastError();
 }
 

@@ -26,7 +26,8 @@ EXPORTS = (
     "esspt_clock", "esspt_set_schedule", "esspt_poll", "esspt_read_schedule", "esspt_read_table",
     "esspt_last_error", "esspt_mf_workspace_bytes", "esspt_mf_scratch_bytes", "esspt_mf_load",
     "esspt_mf_sgd_clock", "esspt_mf_objective", "esspt_mf_minibatch_size", "esspt_mf_export_minibatch",
-    "esspt_mf_stage_minibatch", "esspt_set_profile_events", "esspt_mf_worker_objective_noalloc",
+    "esspt_mf_stage_minibatch", "esspt_mf_stage_bytes", "esspt_set_profile_events",
+    "esspt_mf_worker_objective_noalloc",
     "esspt_mf_sequential_work_bytes", "esspt_mf_sgd_clock_sequential",
 )
 
@@ -87,7 +88,8 @@ def lib() -> ctypes.CDLL:
         "esspt_mf_objective": (ctypes.c_int, [P, I32, ctypes.c_float, P, P, P]),
         "esspt_mf_minibatch_size": (ctypes.c_int, [P, I32, P]),
         "esspt_mf_export_minibatch": (ctypes.c_int, [P, I32, P, P, P, P]),
-        "esspt_mf_stage_minibatch": (ctypes.c_int, [P, I32, P, P, P, P]),
+        "esspt_mf_stage_bytes": (SZ, [P]),
+        "esspt_mf_stage_minibatch": (ctypes.c_int, [P, I32, P, P, P, P, P, SZ, P]),
         "esspt_set_profile_events": (ctypes.c_int, [P, P, P]),
         "esspt_mf_worker_objective_noalloc": (ctypes.c_int, [P, I32, ctypes.c_float, P, P]),
     }
@@ -243,7 +245,9 @@ class Table:
         self._check(L.esspt_mf_load(self._h, di.data_ptr(), dj.data_ptr(), dD.data_ptr(), dm.data_ptr(), n_obs,
                                     dw.data_ptr(), n_users, F, self.mf_workspace.data_ptr(), ws,
                                     scratch.data_ptr(), sc))
-        del scratch
+        del scratch, di, dj, dD, dm, dw
+        # the sort scratch and the input copies can be tens of GB: hand them back
+        torch.cuda.empty_cache()
         self.n_users, self.F, self.n_obs = n_users, F, n_obs
         self._obj_scratch = torch.zeros(2, dtype=torch.float64, device=self.device)
 
@@ -284,10 +288,16 @@ class Table:
                                                     uoff.data_ptr()))
         return u, j, D, uoff
 
-    def mf_stage_minibatch(self, b: int, u, j, D, uoff) -> None:
-        """esspt_mf_stage_minibatch: asynchronous host-to-device copy of minibatch b."""
+    def mf_stage_minibatch(self, b: int, u, j, D, uoff, stream=None) -> None:
+        """esspt_mf_stage_minibatch: asynchronous host-to-device copy of minibatch b
+        on `stream` (a torch.cuda.Stream; None = the table's stream).  The device
+        staging buffer is allocated here (torch) on first use and kept."""
+        need = lib().esspt_mf_stage_bytes(self._h)
+        if getattr(self, "_stage", None) is None or self._stage.numel() < need:
+            self._stage = torch.empty(max(need, 256), dtype=torch.uint8, device=self.device)
+        st = None if stream is None else ctypes.c_void_p(stream.cuda_stream)
         self._check(lib().esspt_mf_stage_minibatch(self._h, b, u.data_ptr(), j.data_ptr(), D.data_ptr(),
-                                                   uoff.data_ptr()))
+                                                   uoff.data_ptr(), self._stage.data_ptr(), self._stage.numel(), st))
 
     def set_profile_events(self, before, after) -> None:
         """esspt_set_profile_events: torch.cuda.Event pair (created) or None."""

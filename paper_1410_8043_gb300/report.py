@@ -23,14 +23,16 @@ import sys
 import numpy as np
 
 
-def run_workload(name: str, clocks: int | None = None) -> dict:
+def run_workload(name, clocks: int | None = None) -> dict:
+    """The report of one workload, given by name or as a gen.workloads.Workload."""
     import torch
 
     from gen import workload
 
     from . import esspt
 
-    w = workload(name)
+    w = workload(name) if isinstance(name, str) else name
+    name = w.name
     C = w.clocks if clocks is None else clocks
     d = w.make_data()
     part = w.partition()

@@ -51,18 +51,19 @@ def test_row_cache_tiny_every_clock(s):
     _run_pair(d, wp, mb, P=w.P, s=s, F=w.F, eta=w.eta, lam=w.lam, cap=w.cap, clocks=w.clocks)
 
 
-@pytest.mark.parametrize("K", [16, 100, 132])
+@pytest.mark.parametrize("K", [16, 48, 100, 132])
 def test_row_cache_row_widths(K):
-    """The generic, one-slice-per-lane and wide-row SGD kernels in row mode."""
+    """The generic, work-list, one-slice-per-lane and wide-row SGD kernels in row mode."""
     d = make_mf_data(n_users=300, n_items=120, n_obs=6000, K=K, seed=K + 1, truth_rank=4, truth_var=0.5,
                      noise_var=0.1, init_var=0.05)
     _run_pair(d, shard_users(300, 5, 1), minibatch_labels(6000, 3, 2), P=5, s=2, F=3, eta=0.02, lam=0.05, cap=0,
               clocks=6)
 
 
-def test_row_cache_heavy_users():
+@pytest.mark.parametrize("K", [32, 64])
+def test_row_cache_heavy_users(K):
     """Users with thousands of entries per minibatch take the chunked path."""
-    d = make_mf_data(n_users=400, n_items=300, n_obs=40000, K=32, seed=9, user_dist="zipf", user_a=1.5,
+    d = make_mf_data(n_users=400, n_items=300, n_obs=40000, K=K, seed=9, user_dist="zipf", user_a=1.5,
                      truth_rank=4, truth_var=0.5, noise_var=0.1, init_var=0.05)
     _run_pair(d, shard_users(400, 3, 8), minibatch_labels(40000, 2, 7), P=3, s=1, F=2, eta=0.002, lam=0.05,
               cap=50, clocks=4)

@@ -49,7 +49,7 @@ def test_sequential_tiny(model):
     _run(d, wp, mb, P=w.P, s=w.s, F=w.F, model=model, eta=w.eta, lam=w.lam, cap=w.cap, clocks=8)
 
 
-@pytest.mark.parametrize("K", [100, 260])
+@pytest.mark.parametrize("K", [64, 100, 260])
 def test_sequential_row_widths_and_cap(K):
     d = make_mf_data(n_users=200, n_items=80, n_obs=5000, K=K, seed=K + 3, truth_rank=4, truth_var=0.5,
                      noise_var=0.1, init_var=0.05)

@@ -1,0 +1,318 @@
+"""Full-size trajectories against the oracle, clock by clock.
+
+Every job below runs one or more GPU tables (through the C-ABI, in the
+launch configuration the benchmark times) next to the fp64 oracle on the
+same seeded inputs, in its own spawned process, so that the oracles of all
+jobs run in parallel on the host cores while the GPU serves every job.
+
+Per clock and per job:
+  * the read-version schedule of every worker, bit for bit;
+  * the clock's squared loss (sum of e^2 over its minibatch at the read
+    versions, the divergence statistic of the D12 reading below), 1e-4
+    relative;
+  * at the job's table clocks: every parameter, |x_gpu - x_oracle| <=
+    1e-4 (1 + |x_oracle|), and whether the clock moved some parameter by
+    more than that tolerance (parity is not vacuous);
+  * at the job's objective clocks: both objectives over all entries, 1e-4
+    relative.
+
+Divergence (Sec. 5: SSP at high staleness may diverge): a clock diverges
+when its squared loss is not finite, exceeds 10 times the previous clock's
+(the onset of a blow-up) or 10^6 times the first clock's.  Parity is checked
+on the clocks before the oracle's first divergent clock, and the GPU's first
+divergent clock must lie within one clock of it.
+
+Jobs:
+  * mid (480k x 18k, 100M entries, K=100, P=32, SSP s=3, cap 20) and
+    mid_essp: all 40 clocks, every table;
+  * the same two at the hot-row cap 190 (robustness to staleness, Sec. 5);
+  * large (10M x 1M, 2B entries, K=64, P=128, SSP s=4): its first 2 clocks;
+  * the staleness / worker sweep on the mid data, s in {0,1,2,4,8} x P in
+    {1,8,64,512} x {SSP, ESSP}, 20 clocks: schedule and loss every clock,
+    tables at clocks 5, 10 and 20 and at every clock on the corners
+    (s in {0, 8}, P in {1, 512}); s = 0 is one oracle for all eight GPU
+    runs (BSP does not depend on P or the model); plus the s = 8 corners at
+    cap 190.
+ESSPT_TRAJ_REPORT=<path> writes every job's per-clock record as JSON lines.
+"""
+import json
+import os
+import shutil
+import tempfile
+import time
+from concurrent.futures import ProcessPoolExecutor
+import multiprocessing as mp
+
+import numpy as np
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-4
+OBJ_RTOL = 1e-4
+DIVERGE = 1e6
+JUMP = 10.0
+_CHUNK = 1 << 23
+
+
+def _violation(g, x):
+    """(max over elements of |g - x| - TOL (1 + |x|), max |g - x|) in fp64,
+    chunked; NaN anywhere counts as +inf."""
+    worst, err = -np.inf, 0.0
+    g = g.reshape(-1)
+    x = x.reshape(-1)
+    for lo in range(0, x.size, _CHUNK):
+        gg = g[lo:lo + _CHUNK].astype(np.float64)
+        xx = x[lo:lo + _CHUNK]
+        d = np.abs(gg - xx)
+        v = float(np.max(d - TOL * (1.0 + np.abs(xx))))
+        worst = max(worst, np.inf if np.isnan(v) else v)
+        m = float(np.max(d))
+        err = max(err, np.inf if np.isnan(m) else m)
+    return worst, err
+
+
+def _moved(x, prev):
+    """Whether some parameter moved by more than the parity tolerance."""
+    x = x.reshape(-1)
+    prev = prev.reshape(-1)
+    for lo in range(0, x.size, _CHUNK):
+        xx = x[lo:lo + _CHUNK]
+        if np.any(np.abs(xx - prev[lo:lo + _CHUNK]) > TOL * (1.0 + np.abs(xx))):
+            return True
+    return False
+
+
+def _diverged(losses):
+    """Whether the last clock of a loss sequence diverged: its loss is not
+    finite, more than JUMP times the previous clock's (the onset of a blow-up,
+    where fp32 rounding grows as fast as the trajectory and parity at 1e-4 is
+    lost within a clock), or more than DIVERGE times the first clock's."""
+    x = losses[-1]
+    if not np.isfinite(x) or x > DIVERGE * losses[0]:
+        return True
+    return len(losses) > 1 and x > JUMP * losses[-2]
+
+
+def _job(spec):
+    """One trajectory: the oracle of the first variant and a GPU table per
+    variant, stepped together.  Runs in a spawned process; returns a record
+    (the checks are asserted by the caller)."""
+    import torch
+
+    from gen import workload
+    from gen.synth import MFData
+    from oracle import Oracle, OracleConfig
+    from paper_1410_8043_gb300 import esspt
+
+    t_start = time.time()
+    variants = [workload(v["base"]).with_(**v["kw"]) for v in spec["variants"]]
+    w0 = variants[0]
+    if spec["data_dir"]:
+        ld = lambda k: np.load(os.path.join(spec["data_dir"], k + ".npy"), mmap_mode="r")  # noqa: E731
+        d = MFData(w0.n_users, w0.n_items, w0.K, ld("i"), ld("j"), ld("D"), ld("L0"), ld("R0"))
+        mb = ld("mb")
+    else:
+        d = w0.make_data()
+        mb = w0.minibatches()
+    gen_s = time.time() - t_start
+    o = Oracle(OracleConfig.from_workload(w0), d.i, d.j, d.D, mb, w0.workers(), d.L0, d.R0)
+    tables = [esspt.Table.for_workload(w, d, (w.workers(), mb)) for w in variants]
+    torch.cuda.empty_cache()
+    losses = [torch.zeros(1, dtype=torch.float64, device="cuda") for _ in variants]
+    C = spec["clocks"]
+    rec = dict(key=spec["key"], clocks=C, gen_s=gen_s, sched_mismatch=[], table=[], objective=[], moved=[],
+               oracle_loss=[], gpu_loss=[[] for _ in variants], div_oracle=None,
+               div_gpu=[None] * len(variants), variants=[w.name for w in variants])
+    x_prev, x_prev_c = None, -1
+    for c in range(1, C + 1):
+        vs = []
+        for k, (w, t) in enumerate(zip(variants, tables)):
+            v, clk = t.read_schedule()
+            assert clk == c
+            vs.append(v)
+            losses[k].zero_()
+            t.mf_sgd_clock(w.eta, w.lam, w.cap, sq_loss=losses[k])
+        o.clock()
+        v_o = o.schedule()
+        ol = o.clock_loss()
+        rec["oracle_loss"].append(ol)
+        for k, w in enumerate(variants):
+            # the oracle's schedule is the first variant's; BSP variants share it
+            if not np.array_equal(vs[k], v_o if w.P == w0.P else np.full(w.P, c - 1, np.int32)):
+                rec["sched_mismatch"].append((w.name, c))
+            gl = float(losses[k].item())
+            rec["gpu_loss"][k].append(gl)
+            if rec["div_gpu"][k] is None and _diverged(rec["gpu_loss"][k]):
+                rec["div_gpu"][k] = c
+        if rec["div_oracle"] is None and _diverged(rec["oracle_loss"]):
+            rec["div_oracle"] = c
+        if rec["div_oracle"] is not None:
+            continue  # parity holds on the clocks before the oracle diverges
+        sparse = spec.get("sparse_clocks", [])
+        want_table = spec["tables"] == "all" or c in spec["tables"]
+        want_obj = c in spec["objective"]
+        if not (want_table or want_obj):
+            continue
+        x = o.table()
+        if want_table:
+            prev = x_prev if x_prev_c == c - 1 else o.table(c - 1)
+            rec["moved"].append((c, _moved(x, prev)))
+            del prev
+        for k, (w, t) in enumerate(zip(variants, tables)):
+            # a variant listed in every_clock is compared at every clock, the others at sparse_clocks
+            if want_table and ("every_clock" not in spec or w.name in spec["every_clock"] or c in sparse):
+                g = t.read_table(c).cpu().numpy()
+                worst, err = _violation(g, x)
+                rec["table"].append((w.name, c, worst, err))
+                del g
+            if want_obj:
+                gs, gp = t.mf_objective(c, w.lam)
+                os_, op = o.objective(c)
+                rec["objective"].append((w.name, c, gs, os_, gp, op))
+        x_prev, x_prev_c = x, c
+        del x
+    for t in tables:
+        t.poll()
+        t.close()
+    del tables, losses, o
+    torch.cuda.empty_cache()
+    rec["seconds"] = time.time() - t_start
+    return rec
+
+
+def _v(base, **kw):
+    return dict(base=base, kw=kw)
+
+
+def _specs(data_dir):
+    from gen.workloads import sweep_workloads
+
+    mid_obj = [1, 20, 40]
+    specs = [
+        dict(key="large", variants=[_v("large")], clocks=2, tables="all", objective=[], data_dir=None),
+        dict(key="mid", variants=[_v("mid")], clocks=40, tables="all", objective=mid_obj),
+        dict(key="mid_essp", variants=[_v("mid_essp")], clocks=40, tables="all", objective=mid_obj),
+        dict(key="mid_cap190", variants=[_v("mid", name="mid_cap190", cap=190)], clocks=40, tables="all",
+             objective=[1, 20]),
+        dict(key="mid_essp_cap190", variants=[_v("mid_essp", name="mid_essp_cap190", cap=190)], clocks=40,
+             tables="all", objective=[1, 20, 40]),
+    ]
+    corner = lambda w: w.s in (0, 8) and w.P in (1, 512)  # noqa: E731
+    sweep = sweep_workloads()
+    bsp = [w for w in sweep if w.s == 0]
+    specs.append(dict(key="sweep_s0", variants=[_v("mid", name=w.name, model=w.model, s=0, P=w.P, clocks=20)
+                                                for w in sorted(bsp, key=lambda w: -w.P)],
+                      clocks=20, tables="all", objective=[20], sparse_clocks=[5, 10, 20],
+                      every_clock=[w.name for w in bsp if corner(w)]))
+    for w in sweep:
+        if w.s == 0:
+            continue
+        specs.append(dict(key=w.name, variants=[_v("mid", name=w.name, model=w.model, s=w.s, P=w.P, clocks=20)],
+                          clocks=20, tables="all" if corner(w) else [5, 10, 20], objective=[20]))
+        if corner(w):
+            specs.append(dict(key=w.name + "_cap190",
+                              variants=[_v("mid", name=w.name + "_cap190", model=w.model, s=w.s, P=w.P, clocks=20,
+                                           cap=190)],
+                              clocks=20, tables="all", objective=[20]))
+    for s in specs:
+        s.setdefault("data_dir", data_dir)
+    return specs
+
+
+@pytest.fixture(scope="module")
+def results():
+    """Submit every job at once; tests collect their own."""
+    from gen import workload
+
+    tmp = tempfile.mkdtemp(prefix="esspt_traj_")
+    w = workload("mid")
+    d = w.make_data()
+    mb = w.partition()[1]
+    for k, arr in dict(i=d.i, j=d.j, D=d.D, mb=mb, L0=d.L0, R0=d.R0).items():
+        np.save(os.path.join(tmp, k + ".npy"), arr)
+    del d, mb
+    specs = _specs(tmp)
+    workers = min(len(specs), max(2, (os.cpu_count() or 4) - 3))
+    ex = ProcessPoolExecutor(max_workers=workers, mp_context=mp.get_context("spawn"))
+    futs = {s["key"]: ex.submit(_job, s) for s in specs}
+    got = {}
+
+    def get(key):
+        if key not in got:
+            got[key] = futs[key].result(timeout=1500)
+        return got[key]
+
+    yield get
+    out = os.environ.get("ESSPT_TRAJ_REPORT")
+    if out:
+        with open(out, "w") as f:
+            for key in futs:
+                if futs[key].done() and not futs[key].cancelled() and futs[key].exception() is None:
+                    f.write(json.dumps(futs[key].result()) + "\n")
+    ex.shutdown(wait=True, cancel_futures=True)
+    shutil.rmtree(tmp, ignore_errors=True)
+
+
+def _check(rec, want_div=None, moved_share=0.8):
+    key = rec["key"]
+    assert not rec["sched_mismatch"], (key, rec["sched_mismatch"][:5])
+    C = rec["div_oracle"] or rec["clocks"] + 1
+    for name, c, worst, err in rec["table"]:
+        assert worst <= 0.0, f"{key}/{name} clock {c}: max |err| {err:.3e}"
+    for name, c, gs, os_, gp, op in rec["objective"]:
+        assert abs(gs - os_) <= OBJ_RTOL * abs(os_) and abs(gp - op) <= OBJ_RTOL * abs(op), (key, name, c, gs, os_)
+    for k, name in enumerate(rec["variants"]):
+        for c in range(1, min(C, rec["clocks"] + 1)):
+            gl, ol = rec["gpu_loss"][k][c - 1], rec["oracle_loss"][c - 1]
+            assert abs(gl - ol) <= OBJ_RTOL * abs(ol), (key, name, c, gl, ol)
+        dg, do = rec["div_gpu"][k], rec["div_oracle"]
+        if do is None:
+            assert dg is None or dg == rec["clocks"], (key, name, dg)
+        else:
+            assert dg is not None and abs(dg - do) <= 1, (key, name, dg, do)
+    if want_div is not None:
+        assert (rec["div_oracle"] is not None) == want_div, (key, rec["div_oracle"])
+    checked = [m for c, m in rec["moved"]]
+    if checked:  # parity is not vacuous: most clocks move parameters by more than the tolerance
+        assert sum(checked) >= moved_share * len(checked), (key, rec["moved"])
+
+
+@pytest.mark.parametrize("key", ["mid", "mid_essp"])
+def test_mid_every_clock(results, key):
+    rec = results(key)
+    _check(rec, want_div=False)
+    assert len([t for t in rec["table"]]) == 40
+
+
+def test_cap190_ssp_diverges_essp_stays_stable(results):
+    """Sec. 5, robustness to staleness: at the larger step cap SSP s=3
+    diverges within 40 clocks while ESSP converges; the GPU follows the
+    oracle up to the divergence and flags it within one clock."""
+    ssp = results("mid_cap190")
+    essp = results("mid_essp_cap190")
+    _check(ssp)
+    _check(essp, want_div=False)
+    assert ssp["div_oracle"] is not None, "SSP s=3 at cap 190 did not diverge in 40 clocks"
+
+
+def test_large_first_clocks(results):
+    rec = results("large")
+    _check(rec, want_div=False)
+    assert [c for _, c, _, _ in rec["table"]] == [1, 2]
+
+
+def test_sweep_every_combination(results):
+    from gen.workloads import sweep_workloads
+
+    keys = ["sweep_s0"] + [w.name for w in sweep_workloads() if w.s > 0]
+    for key in keys:
+        _check(results(key))
+
+
+def test_sweep_s8_corners_at_cap190(results):
+    from gen.workloads import sweep_workloads
+
+    for w in sweep_workloads():
+        if w.s == 8 and w.P in (1, 512):
+            _check(results(w.name + "_cap190"))

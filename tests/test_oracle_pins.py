@@ -205,6 +205,18 @@ def test_essp_stationary_staleness_closed_form():
     assert abs(st.mean() - 0.327729) < 5 * st.std() / np.sqrt(n) * 3
 
 
+def test_essp_delay_thresholds_exact():
+    """The ESSP delay rule's 32-bit thresholds are floor(0.3^k 2^32) for the
+    Geometric(0.7) delay (failures before the first success), computed here
+    in exact rational arithmetic."""
+    from oracle import essp_thresholds
+
+    cfg = OracleConfig(n_users=1, n_items=1, K=1, P=1, s=3, F=1, model="essp", essp_p=0.7, essp_max_delay=3)
+    want = [int(Fraction(3, 10) ** k * 2 ** 32) for k in (1, 2, 3)]
+    assert want == [1288490188, 386547056, 115964116]
+    assert essp_thresholds(cfg) == want
+
+
 def test_essp_clamped_by_s():
     """For s < 3 the delay is clamped to s, so ESSP never leaves the SSP window."""
     for s in (1, 2):
