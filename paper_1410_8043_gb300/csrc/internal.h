@@ -87,7 +87,8 @@ struct SgdArgs {
                             // (slot * n_rows + N + item) of the item's cached version
   const float* rec_D;       // value of each entry of minibatch b
   const int32_t* rec_dst;   // replica row in dR that each entry's item update adds into
-  const int32_t* item_rep;  // [M+1] first replica row of each item in dR
+  const int32_t* item_rep;  // [M+1] prefix of extra replicas: replica 0 of item j is row j of dR,
+                            // replica r > 0 row M + item_rep[j] + r - 1
   float* dR;                // item delta replicas (all zero between clocks)
   int32_t dR_ld;            // float4 per dR row (K rounded up to whole 32-byte sectors)
   float eta, lambda;

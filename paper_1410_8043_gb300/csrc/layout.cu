@@ -144,7 +144,8 @@ __global__ void heavy_kernel(const int64_t* __restrict__ choff, const int32_t* _
   }
 }
 
-// Replica count of every item from its largest minibatch count.
+// Extra replica rows of every item (replicas - 1) from its largest minibatch
+// count.  Replica 0 of item j is row j of dR; the extra ones follow all items.
 __global__ void item_reps_kernel(const int32_t* __restrict__ item_cnt, int64_t n_items, int32_t F,
                                  int32_t* __restrict__ reps) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -155,22 +156,24 @@ __global__ void item_reps_kernel(const int32_t* __restrict__ item_cnt, int64_t n
     }
     int32_t mx = 0;
     for (int32_t b = 0; b < F; ++b) mx = max(mx, item_cnt[(int64_t)b * n_items + j]);
-    reps[j] = item_reps(mx);
+    reps[j] = item_reps(mx) - 1;
   }
 }
 
 // Replica row of every entry's item update: entry t (position within its
-// minibatch) of item j adds into row item_rep[j] + (t mod replicas of j).
+// minibatch) of item j adds into replica (t mod replicas of j): replica 0 is
+// row j, replica r > 0 row n_items + item_rep[j] + r - 1.
 __global__ void dst_kernel(const uint32_t* __restrict__ key, const int64_t* __restrict__ mb_base,
                            const int32_t* __restrict__ rec_j, const int32_t* __restrict__ item_rep, int64_t n_obs,
-                           int64_t n_users, int32_t* __restrict__ rec_dst) {
+                           int64_t n_users, int64_t n_items, int32_t* __restrict__ rec_dst) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < n_obs; k += stride) {
     const int64_t b = (int64_t)key[k] / n_users;
     const int64_t t = k - mb_base[b];
     const int32_t j = rec_j[k];
-    const int32_t r0 = item_rep[j], r1 = item_rep[j + 1];
-    rec_dst[k] = r0 + (int32_t)(t & (int64_t)(r1 - r0 - 1));
+    const int32_t e0 = item_rep[j], e1 = item_rep[j + 1];  // extra replicas of j: e1 - e0 (reps - 1)
+    const int32_t r = (int32_t)(t & (int64_t)(e1 - e0));    // reps is a power of two
+    rec_dst[k] = r == 0 ? j : (int32_t)(n_items + e0 + r - 1);
   }
 }
 
@@ -256,7 +259,7 @@ int64_t layout_max_chunks(int64_t n_obs, int32_t F, int64_t n_users, bool light_
 
 int64_t layout_max_heavy(int64_t n_obs, int32_t F) { return n_obs / (kHeavy + 1) + F + 1; }
 
-// sum over items of replicas: n_items + sum (reps - 1), and reps - 1 < 3 mx / (2 kItemRep).
+// Replica rows: one per item plus the extra ones, sum (reps - 1) with reps - 1 < 3 mx / (2 kItemRep).
 int64_t layout_max_item_reps(int64_t n_obs, int64_t n_items) { return n_items + 3 * n_obs / (2 * kItemRep) + 2; }
 
 // Extra replica rows of heavy users: reps - 1 < 3 nch / (2 kUserRep), sum nch < 2 n_obs / kChunk.
@@ -320,7 +323,7 @@ cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st) {
     return e;
   if (b.n_obs == 0) return cudaSuccess;
   dst_kernel<<<blocks_for(b.n_obs), 256, 0, st>>>(key_out, b.mb_base, b.rec_j, b.item_rep, b.n_obs, b.n_users,
-                                                  b.rec_dst);
+                                                  b.n_items, b.rec_dst);
   return cudaGetLastError();
 }
 

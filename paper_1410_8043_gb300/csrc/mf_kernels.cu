@@ -526,17 +526,20 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
 
 // Rows of 36..64 values (9..16 float4 slices) on the work-list path.
 //
-// sgd_work16_kernel: one warp per work item of minibatch b, either a user
-// with 1..kHeavy entries (written once: L^c = L^base + eta s sum_k(e_k R_j -
-// lambda L_i)) or a 64-entry chunk of a heavy user (its unscaled partial sum
-// goes into the chunk's replica row of dL, merged by heavy_merge_kernel).
-// Both halves of the warp hold the item's row L_i (lane l owns slice l mod
-// 16); a step takes 8 entries, half h the entries 2m + h (m = 0..3), so each
-// gather instruction brings two item rows.  A transposing butterfly over the
-// 16 lanes of a half (4 shuffles) leaves entry 2m + h's dot product on lanes
-// 4m .. 4m+3 of half h.  The item's rows at the read and base versions are
-// staged in shared memory one item ahead by cp.async, and each warp walks one
-// contiguous range of items, balanced by entries plus kItemCost per item.
+// sgd_work16_kernel: one half-warp per work item of minibatch b, the two
+// halves of a warp on consecutive items in lockstep.  An item is either a
+// user with 1..kHeavy entries (written once: L^c = L^base + eta s sum_k(e_k
+// R_j - lambda L_i)) or a 64-entry chunk of a heavy user (its unscaled
+// partial sum goes into the chunk's replica row of dL, merged by
+// heavy_merge_kernel).  Lane l owns slice l mod 16 of its half's row L_i; a
+// step takes 4 entries per half, so each gather instruction brings two item
+// rows, and a transposing butterfly over the 16 lanes of a half (4 shuffles)
+// leaves entry e's dot product on lanes 4e .. 4e+3.  Items are mostly users
+// with a few entries, so pairing them keeps most gather slots busy and
+// shares the per-item work (metadata, staging, the row store) between two
+// items.  The items' rows at the read and base versions are staged in shared
+// memory one pair ahead by cp.async, and each warp walks one contiguous range
+// of items, balanced by entries plus kItemCost per item.
 #ifndef ESSPT_WORK16_MINB
 #define ESSPT_WORK16_MINB 3
 #endif
@@ -544,14 +547,16 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
 #define ESSPT_W16_ITEMCOST 6
 #endif
 constexpr int32_t kItemCost = ESSPT_W16_ITEMCOST;
-constexpr int kW16Unit = 16;
+constexpr int kW16Unit = 16;      // items per metadata unit (8 pairs)
+constexpr int32_t kNoItem = -2;   // metadata of a slot past the warp's range
 
 __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(ChunkArgs c) {
   const SgdArgs& a = c.a;
-  __shared__ __align__(16) float4 stage[8][2][2][16];  // [warp][buffer][read row, base row][slice]
+  __shared__ __align__(16) float4 stage[8][2][2][32];  // [warp][buffer][read row, base row][half * 16 + slice]
   const int lane = threadIdx.x & 31;
   const int wib = threadIdx.x >> 5;
-  const int h = lane >> 4;      // half: entries 2m + h of a step
+  const int h = lane >> 4;      // half: its own item
+  const int hb = lane & 16;     // first lane of the half
   const int r = lane & 15;      // slice of the row this lane owns
   const int32_t K4 = a.K >> 2;
   const bool on = r < K4;
@@ -605,12 +610,12 @@ __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(Chun
   }
 
   // Item metadata: the current unit in lanes [0, 16), the next in [16, 32).
-  int4 m_it = make_int4(0, 0, 0, 0);
+  int4 m_it = make_int4(0, 0, 0, kNoItem);
   int32_t m_vs = 0;
   auto load_meta = [&](int64_t first, int lo) {
     if (lane >= lo && lane < lo + kW16Unit) {
       const int64_t x = first + (lane - lo);
-      m_it = make_int4(0, 0, 0, 0);
+      m_it = make_int4(0, 0, 0, kNoItem);
       m_vs = 0;
       if (x < ib) {
         m_it = __ldg(c.chunk + x);
@@ -618,66 +623,74 @@ __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(Chun
       }
     }
   };
-  // Stage item ml's rows: lanes [0, 16) its read-version row, lanes [16, 32)
-  // its base row (only a light user whose read version is not the base).
-  auto stage_item = [&](int ml, int bb) {
-    const int32_t u = __shfl_sync(0xffffffffu, m_it.x, ml);
-    const int32_t dst = __shfl_sync(0xffffffffu, m_it.w, ml);
-    const int32_t vs = __shfl_sync(0xffffffffu, m_vs, ml);
-    const bool same = vs == a.slot_base;
+  // Stage the pair whose first item's metadata sits in lane ml: half h its
+  // item's read-version row and, for a user item whose read version is not
+  // the base, its base row.
+  auto stage_pair = [&](int ml, int bb) {
+    const int32_t u = __shfl_sync(0xffffffffu, m_it.x, ml + h);
+    const int32_t dst = __shfl_sync(0xffffffffu, m_it.w, ml + h);
+    const int32_t vs = __shfl_sync(0xffffffffu, m_vs, ml + h);
     const int64_t row = (int64_t)u * K4 + (on ? r : 0);
-    if (h == 0)
-      cp_async16_hint(&stage[wib][bb][0][r], ring4 + (int64_t)vs * slot4 + row, on, pol);
-    else
-      cp_async16_hint(&stage[wib][bb][1][r], base4 + row, on && dst < 0 && !same, pol);
+    cp_async16_hint(&stage[wib][bb][0][lane], ring4 + (int64_t)vs * slot4 + row, on && dst != kNoItem, pol);
+    cp_async16_hint(&stage[wib][bb][1][lane], base4 + row, on && dst == -1 && vs != a.slot_base, pol);
     cp_async_commit();
   };
 
   load_meta(ia, 0);
   load_meta((int64_t)ia + kW16Unit, kW16Unit);
-  Window<32> win;
-  stage_item(0, 0);
-  win.reload(a, __shfl_sync(0xffffffffu, m_it.y, 0), lane);
+  stage_pair(0, 0);
   int bb = 0;
+  // This half's window of 16 entries: lane hb + i holds entry W + i.
+  int32_t W = 0, cj = 0, cdst = 0;
+  float cd = 0.f;
   for (int64_t x0 = ia; x0 < ib; x0 += kW16Unit) {
     const int32_t nloc = (int32_t)min((int64_t)kW16Unit, (int64_t)ib - x0);
-    for (int32_t t = 0; t < nloc; ++t, bb ^= 1) {
+    for (int32_t t = 0; 2 * t < nloc; ++t, bb ^= 1) {
       cp_async_wait_all();
       __syncwarp();
-      if (t + 1 < nloc) {
-        stage_item(t + 1, bb ^ 1);
+      if (2 * t + 2 < nloc) {
+        stage_pair(2 * t + 2, bb ^ 1);
       } else if (x0 + kW16Unit < ib) {
-        stage_item(kW16Unit, bb ^ 1);
+        stage_pair(kW16Unit, bb ^ 1);
       }
-      const int32_t u = __shfl_sync(0xffffffffu, m_it.x, t);
-      const int32_t beg = __shfl_sync(0xffffffffu, m_it.y, t);
-      const int32_t end = __shfl_sync(0xffffffffu, m_it.z, t);
-      const int32_t dst = __shfl_sync(0xffffffffu, m_it.w, t);
-      const int32_t vs = __shfl_sync(0xffffffffu, m_vs, t);
-      const float4 Lv = stage[wib][bb][0][r];
+      const int src = 2 * t + h;
+      const int32_t u = __shfl_sync(0xffffffffu, m_it.x, src);
+      const int32_t beg = __shfl_sync(0xffffffffu, m_it.y, src);
+      const int32_t dst = __shfl_sync(0xffffffffu, m_it.w, src);
+      const int32_t z = __shfl_sync(0xffffffffu, m_it.z, src);  // every lane takes part in every shuffle
+      const int32_t end = dst == kNoItem ? beg : z;
+      const int32_t vs = __shfl_sync(0xffffffffu, m_vs, src);
+      const int32_t n = end - beg;
+      const float4 Lv = stage[wib][bb][0][lane];
       // Lanes past the row end read slice 0 of the item rows; their staged L is
       // zero, so they add nothing to the dot products.
       const float4* Rq =
           (a.row_mode ? ring4 : ring4 + (int64_t)vs * slot4 + (int64_t)a.n_users * K4) + (on ? r : 0);
       float4 gL = f4_zero();
-      auto step = [&](auto full_tag, int32_t tt, int32_t cnt) {
+      W = beg;
+      load_entry(a, W + r, cj, cd, cdst);
+      const int32_t nsteps = (n + 3) >> 2;
+      const int32_t steps = max(nsteps, __shfl_xor_sync(0xffffffffu, nsteps, 16));
+      // One step: entries tt .. tt+cnt-1 of this half's item (cnt <= 4, 0 once
+      // the item is done while the other half's continues).  Compiled twice:
+      // for steps where both halves have 4 entries, whose loads need no
+      // predicate, and for the others.
+      auto step = [&](auto full_tag, int32_t w0, int32_t cnt) {
         constexpr bool kFull = decltype(full_tag)::value;
-        const int w0 = tt - win.W;
         float4 R[4];
         int32_t dsts[4];
         float p[4];
 #pragma unroll
-        for (int m = 0; m < 4; ++m) {
-          const int k = 2 * m + h;
-          const int src = kFull ? w0 + k : min(w0 + k, 31);
-          const int32_t j = __shfl_sync(0xffffffffu, win.cj, src);
-          dsts[m] = __shfl_sync(0xffffffffu, win.cdst, src);
-          R[m] = (kFull || k < cnt) ? __ldg(Rq + j * K4) : f4_zero();
-          p[m] = dot4(Lv, R[m]);
+        for (int e = 0; e < 4; ++e) {
+          const int sl = hb + (kFull ? w0 + e : min(w0 + e, 15));
+          const int32_t j = __shfl_sync(0xffffffffu, cj, sl);
+          dsts[e] = __shfl_sync(0xffffffffu, cdst, sl);
+          R[e] = (kFull || e < cnt) ? __ldg(Rq + j * K4) : f4_zero();
+          p[e] = dot4(Lv, R[e]);
         }
         // Transposing butterfly over the 16 lanes of a half: bit 3 of the
         // lane keeps entries {0,1} or {2,3}, bit 2 one of the pair, bits 1
-        // and 0 sum; lanes 4m .. 4m+3 end with entry 2m + h's dot product.
+        // and 0 sum; lanes 4e .. 4e+3 end with entry e's dot product.
         const bool b3 = r & 8, b2 = r & 4;
         float k0 = b3 ? p[2] : p[0], k1 = b3 ? p[3] : p[1];
         k0 += __shfl_xor_sync(0xffffffffu, b3 ? p[0] : p[2], 8);
@@ -686,49 +699,47 @@ __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(Chun
         dot += __shfl_xor_sync(0xffffffffu, b2 ? k0 : k1, 4);
         dot += __shfl_xor_sync(0xffffffffu, dot, 2);
         dot += __shfl_xor_sync(0xffffffffu, dot, 1);
-        const int kq = 2 * (r >> 2) + h;  // the entry this lane's dot product belongs to
-        const float dq = __shfl_sync(0xffffffffu, win.cd, kFull ? w0 + kq : min(w0 + kq, 31));
+        const int kq = r >> 2;  // the entry this lane's dot product belongs to
+        const float dq = __shfl_sync(0xffffffffu, cd, hb + (kFull ? w0 + kq : min(w0 + kq, 15)));
         const float eq = (kFull || kq < cnt) ? dq - dot : 0.f;
         if ((r & 3) == 0) loss += eq * eq;
 #pragma unroll
-        for (int m = 0; m < 4; ++m) {
-          const float e = __shfl_sync(0xffffffffu, eq, (lane & 16) + 4 * m);
-          const float4 rr = R[m];
-          gL.x += e * rr.x;
-          gL.y += e * rr.y;
-          gL.z += e * rr.z;
-          gL.w += e * rr.w;
-          red_add_v4_if(dRq + dsts[m] * a.dR_ld,
-                        make_float4(e * Lv.x - a.lambda * rr.x, e * Lv.y - a.lambda * rr.y,
-                                    e * Lv.z - a.lambda * rr.z, e * Lv.w - a.lambda * rr.w),
-                        on && (kFull || 2 * m + h < cnt));
+        for (int e = 0; e < 4; ++e) {
+          const float ev = __shfl_sync(0xffffffffu, eq, hb + 4 * e);
+          const float4 rr = R[e];
+          gL.x += ev * rr.x;
+          gL.y += ev * rr.y;
+          gL.z += ev * rr.z;
+          gL.w += ev * rr.w;
+          red_add_v4_if(dRq + dsts[e] * a.dR_ld,
+                        make_float4(ev * Lv.x - a.lambda * rr.x, ev * Lv.y - a.lambda * rr.y,
+                                    ev * Lv.z - a.lambda * rr.z, ev * Lv.w - a.lambda * rr.w),
+                        on && (kFull || e < cnt));
         }
       };
-      for (int32_t tt = beg; tt < end;) {
-        win.cover(a, tt, lane);
-        const int32_t cnt = min(8, min(end - tt, win.W + 32 - tt));
-        if (cnt == 8) {
-          step(std::true_type{}, tt, cnt);
-        } else {
-          step(std::false_type{}, tt, cnt);
+      for (int32_t sidx = 0; sidx < steps; ++sidx) {
+        const int32_t tt = beg + 4 * sidx;
+        const int32_t cnt = max(0, min(4, end - tt));
+        if (__any_sync(0xffffffffu, cnt > 0 && tt + cnt > W + 16)) {  // slide a half's window
+          if (cnt > 0 && tt + cnt > W + 16) {
+            W = tt;
+            load_entry(a, W + r, cj, cd, cdst);
+          }
         }
-        tt += cnt;
+        if (__all_sync(0xffffffffu, cnt == 4)) {
+          step(std::true_type{}, tt - W, 4);
+        } else {
+          step(std::false_type{}, tt - W, cnt);
+        }
       }
-      // both halves' sums, then the -lambda L_i term of every entry
-      gL.x += __shfl_xor_sync(0xffffffffu, gL.x, 16);
-      gL.y += __shfl_xor_sync(0xffffffffu, gL.y, 16);
-      gL.z += __shfl_xor_sync(0xffffffffu, gL.z, 16);
-      gL.w += __shfl_xor_sync(0xffffffffu, gL.w, 16);
-      const int32_t n = end - beg;
       const float4 g = f4_axpy(-(float)n * a.lambda, Lv, gL);
       if (dst >= 0) {  // a heavy user's chunk: unscaled partial sum into its replica row
-        if (h == 0 && on) red_add_v4(dL4 + (int64_t)dst * K4 + r, g);
-      } else {
-        const bool same = vs == a.slot_base;
-        const float4 lb = same ? Lv : stage[wib][bb][1][r];
+        if (on) red_add_v4(dL4 + (int64_t)dst * K4 + r, g);
+      } else if (dst == -1) {
+        const float4 lb = vs == a.slot_base ? Lv : stage[wib][bb][1][lane];
         float sc = a.eta;
         if (a.cap > 0 && n > a.cap) sc = a.eta * capped_scale(a.cap, n);
-        st_stream_if(outq + (int64_t)u * K4 + r, f4_axpy(sc, g, lb), pol, h == 0 && on);
+        st_stream_if(outq + (int64_t)u * K4 + r, f4_axpy(sc, g, lb), pol, on);
       }
     }
     m_it.x = __shfl_down_sync(0xffffffffu, m_it.x, kW16Unit);
@@ -893,9 +904,11 @@ __global__ void __launch_bounds__(256) heavy_merge_kernel(HeavyMergeArgs a) {
 
 // Clock() merge of the item rows (Sec. 2.1 additive updates, Sec. 4 server
 // clock): R^c_j = R^base_j + eta s_j sum of j's replica rows; replicas
-// cleared.  One thread per (item, float4 slice).  With do_schedule the first
-// P threads also compute the next clock's read versions (the SGD kernels of
-// this clock, the only readers of v, have finished).
+// cleared.  One thread per (item, float4 slice).  Replica 0 of item j is row
+// j of dR, so the common single-replica item needs no index load before its
+// data loads: every load of a thread is issued at once.  With do_schedule the
+// first P threads also compute the next clock's read versions (the SGD
+// kernels of this clock, the only readers of v, have finished).
 __global__ void __launch_bounds__(256) item_merge_kernel(ItemMergeArgs a) {
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t nth = (int64_t)gridDim.x * blockDim.x;
@@ -905,15 +918,48 @@ __global__ void __launch_bounds__(256) item_merge_kernel(ItemMergeArgs a) {
   const int64_t slot4 = a.n_rows * K4;
   float4* ring4 = reinterpret_cast<float4*>(a.ring);
   float4* dR4 = reinterpret_cast<float4*>(a.dR);
+  // n_items * K/4 < 2^31 (checked at load), so the (item, slice) split is a
+  // 32-bit division
   const int64_t total = (int64_t)a.n_items * K4;
-  for (int64_t x = tid; x < total; x += nth) {
-    const int64_t j = x / K4;
-    const int32_t q = (int32_t)(x - j * K4);
-    const int32_t r0 = __ldg(a.item_rep + j), r1 = __ldg(a.item_rep + j + 1);
-    const float sc = a.eta * cap_scale(a.cap, __ldg(a.item_cnt + j));
-    const float4 acc = sum_and_clear(dR4 + (int64_t)r0 * a.dR_ld + q, r1 - r0, a.dR_ld);
-    const int64_t row = ((int64_t)a.n_users + j) * K4 + q;
-    ring4[(int64_t)a.slot_out * slot4 + row] = f4_axpy(sc, acc, ring4[(int64_t)a.slot_base * slot4 + row]);
+#ifndef ESSPT_MERGE_U
+#define ESSPT_MERGE_U 8
+#endif
+  constexpr int U = ESSPT_MERGE_U;  // (item, slice) pairs per thread per round, loads of all in flight
+  for (int64_t x0 = tid; x0 < total; x0 += U * nth) {
+    float4 first[U], base[U];
+    int32_t e0[U], e1[U], cnt[U];
+    int64_t row[U], dofs[U];
+#pragma unroll
+    for (int k = 0; k < U; ++k) {
+      const int64_t x = min(x0 + k * nth, total - 1);
+      const uint32_t j = (uint32_t)x / (uint32_t)K4;
+      const int32_t q = (int32_t)((uint32_t)x - j * (uint32_t)K4);
+      row[k] = ((int64_t)a.n_users + j) * K4 + q;
+      dofs[k] = (int64_t)j * a.dR_ld + q;
+#ifdef ESSPT_MERGE_STREAM
+      const uint64_t pol = policy_evict_first();
+      first[k] = ld_stream(dR4 + dofs[k], pol);
+      base[k] = ld_stream(ring4 + (int64_t)a.slot_base * slot4 + row[k], pol);
+#else
+      first[k] = dR4[dofs[k]];
+      base[k] = ring4[(int64_t)a.slot_base * slot4 + row[k]];
+#endif
+      e0[k] = __ldg(a.item_rep + j);
+      e1[k] = __ldg(a.item_rep + j + 1);
+      cnt[k] = __ldg(a.item_cnt + j);
+    }
+#pragma unroll
+    for (int k = 0; k < U; ++k) {
+      if (x0 + k * nth >= total) break;
+      dR4[dofs[k]] = f4_zero();
+      float4 acc = first[k];
+      if (e1[k] > e0[k]) {
+        const int32_t q = (int32_t)(dofs[k] % a.dR_ld);
+        acc = f4_add(acc, sum_and_clear(dR4 + ((int64_t)a.n_items + e0[k]) * a.dR_ld + q, e1[k] - e0[k], a.dR_ld));
+      }
+      const float sc = a.eta * cap_scale(a.cap, cnt[k]);
+      ring4[(int64_t)a.slot_out * slot4 + row[k]] = f4_axpy(sc, acc, base[k]);
+    }
   }
 }
 
@@ -999,13 +1045,22 @@ cudaError_t launch_sgd_chunks(const ChunkArgs& c, cudaStream_t st) { return disp
 
 // One resident wave of sgd_work16_kernel; its warps balance the items among
 // themselves.
+#ifndef ESSPT_W16_CARVEOUT
+#define ESSPT_W16_CARVEOUT 25
+#endif
 cudaError_t launch_sgd_work16(const ChunkArgs& c, cudaStream_t st) {
   if (c.n_chunks <= 0) return cudaSuccess;
   static int per_sm = 0;
-  if (per_sm == 0 &&
-      (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sgd_work16_kernel, 256, 0) != cudaSuccess ||
-       per_sm <= 0))
-    per_sm = 1;
+  if (per_sm == 0) {
+    // The smallest shared-memory carveout that holds the resident blocks'
+    // staging buffers (percent of the maximum): the rest of the SM's memory is
+    // L1, which keeps the popular item rows.
+    if (ESSPT_W16_CARVEOUT >= 0)
+      cudaFuncSetAttribute(sgd_work16_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, ESSPT_W16_CARVEOUT);
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sgd_work16_kernel, 256, 0) != cudaSuccess ||
+        per_sm <= 0)
+      per_sm = 1;
+  }
   sgd_work16_kernel<<<grid_for((c.n_chunks + kW16Unit - 1) / kW16Unit, 8, std::min(per_sm, kWorkBlocksPerSm)), 256,
                       0, st>>>(c);
   return cudaGetLastError();
@@ -1036,7 +1091,7 @@ cudaError_t launch_item_merge(const ItemMergeArgs& a, cudaStream_t st) {
   // One thread per (item, slice): every thread's loads are independent, so
   // the whole merge is one set of in-flight requests rather than a
   // grid-stride chain of dependent ones.
-  const int64_t blocks = std::min<int64_t>((work + 255) / 256, (int64_t)1 << 30);
+  const int64_t blocks = std::min<int64_t>((work + 255 * ESSPT_MERGE_U) / (256 * ESSPT_MERGE_U), (int64_t)1 << 30);
   item_merge_kernel<<<(unsigned)blocks, 256, 0, st>>>(a);
   return cudaGetLastError();
 }

@@ -279,11 +279,18 @@ class Table:
         self._check(lib().esspt_mf_minibatch_size(self._h, b, ctypes.byref(n)))
         return n.value
 
-    def mf_export_minibatch(self, b: int, pin: bool = True):
-        """esspt_mf_export_minibatch: (u, j, D, uoff) host tensors of minibatch b."""
+    def mf_export_minibatch(self, b: int, pin: bool = True, out=None):
+        """esspt_mf_export_minibatch: (u, j, D, uoff) host tensors of minibatch b,
+        written into `out` (four contiguous host tensors of the right sizes) if given."""
         n = self.mf_minibatch_size(b)
-        mk = lambda k, dt: torch.empty(k, dtype=dt, pin_memory=pin)  # noqa: E731
-        u, j, D, uoff = mk(n, torch.int32), mk(n, torch.int32), mk(n, torch.float32), mk(self.n_users + 1, torch.int32)
+        if out is not None:
+            u, j, D, uoff = out
+            assert u.numel() == n and j.numel() == n and D.numel() == n and uoff.numel() == self.n_users + 1
+            assert u.dtype == j.dtype == uoff.dtype == torch.int32 and D.dtype == torch.float32
+            assert all(x.is_contiguous() and x.device.type == "cpu" for x in out)
+        else:
+            mk = lambda k, dt: torch.empty(k, dtype=dt, pin_memory=pin)  # noqa: E731
+            u, j, D, uoff = mk(n, torch.int32), mk(n, torch.int32), mk(n, torch.float32), mk(self.n_users + 1, torch.int32)
         self._check(lib().esspt_mf_export_minibatch(self._h, b, u.data_ptr(), j.data_ptr(), D.data_ptr(),
                                                     uoff.data_ptr()))
         return u, j, D, uoff

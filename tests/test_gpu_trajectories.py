@@ -30,9 +30,9 @@ Jobs:
   * the staleness / worker sweep on the mid data, s in {0,1,2,4,8} x P in
     {1,8,64,512} x {SSP, ESSP}, 20 clocks: schedule and loss every clock,
     tables at clocks 5, 10 and 20 and at every clock on the corners
-    (s in {0, 8}, P in {1, 512}); s = 0 is one oracle for all eight GPU
-    runs (BSP does not depend on P or the model); plus the s = 8 corners at
-    cap 190.
+    (s in {0, 8}, P in {1, 512}); s = 0 is one oracle for the four GPU
+    runs of each model (BSP does not depend on P); plus the s = 8 corners
+    at cap 190.
 ESSPT_TRAJ_REPORT=<path> writes every job's per-clock record as JSON lines.
 """
 import json
@@ -200,11 +200,13 @@ def _specs(data_dir):
     ]
     corner = lambda w: w.s in (0, 8) and w.P in (1, 512)  # noqa: E731
     sweep = sweep_workloads()
-    bsp = [w for w in sweep if w.s == 0]
-    specs.append(dict(key="sweep_s0", variants=[_v("mid", name=w.name, model=w.model, s=0, P=w.P, clocks=20)
-                                                for w in sorted(bsp, key=lambda w: -w.P)],
-                      clocks=20, tables="all", objective=[20], sparse_clocks=[5, 10, 20],
-                      every_clock=[w.name for w in bsp if corner(w)]))
+    for model in ("ssp", "essp"):
+        bsp = [w for w in sweep if w.s == 0 and w.model == model]
+        specs.append(dict(key=f"sweep_{model}_s0",
+                          variants=[_v("mid", name=w.name, model=w.model, s=0, P=w.P, clocks=20)
+                                    for w in sorted(bsp, key=lambda w: -w.P)],
+                          clocks=20, tables="all", objective=[20], sparse_clocks=[5, 10, 20],
+                          every_clock=[w.name for w in bsp if corner(w)]))
     for w in sweep:
         if w.s == 0:
             continue
@@ -305,7 +307,7 @@ def test_large_first_clocks(results):
 def test_sweep_every_combination(results):
     from gen.workloads import sweep_workloads
 
-    keys = ["sweep_s0"] + [w.name for w in sweep_workloads() if w.s > 0]
+    keys = ["sweep_ssp_s0", "sweep_essp_s0"] + [w.name for w in sweep_workloads() if w.s > 0]
     for key in keys:
         _check(results(key))
 
