@@ -176,7 +176,13 @@ class FloorModel:
     (v != c-1) by a user with entries; each distinct (item, stale version)
     row read.  Item rows of version c-1 count as resident (the previous
     clock's merge just wrote them).  Counted with torch on `device` (the
-    distinct pairs by sorting), one minibatch at a time."""
+    distinct pairs by sorting), one minibatch at a time.
+
+    On the work-list path (32 < K <= 64) an idle user row unchanged over the
+    last s+2 clocks is not merged (its ring slot already holds it), and each
+    user has a 4-byte change-clock word, read for idle users and written for
+    active ones.  `bytes` must then see every clock from the table's version
+    0 in order."""
 
     def __init__(self, w, data, wp, mb, device="cpu"):
         import torch
@@ -189,6 +195,9 @@ class FloorModel:
         self.wp = torch.as_tensor(np.ascontiguousarray(wp)).to(self.dev).long()
         self._b = None
         self._per_b = {}
+        self.skip = 32 < w.K <= 64
+        self.chg = torch.zeros(w.n_users, dtype=torch.int64, device=self.dev) if self.skip else None
+        self.last_c = 0
 
     def _minibatch(self, b):
         """(entries, worker of each user with entries, distinct worker*M + item
@@ -203,7 +212,7 @@ class FloorModel:
             uw = self.wp[users]
             pj = torch.unique(self.wp[ui] * self.w.n_items + jj)
             heavy = bool(cnt.numel() and int(cnt.max()) > 96)
-            self._cache = (int(idx.numel()), uw, pj, heavy)
+            self._cache = (int(idx.numel()), uw, pj, heavy, users)
             self._b = b
             del idx, ui, jj, users, cnt
         return self._cache
@@ -220,7 +229,7 @@ class FloorModel:
 
         w = self.w
         b = (c - 1) % w.F
-        n, uw, pj, heavy = self._minibatch(b)
+        n, uw, pj, heavy, active = self._minibatch(b)
         self._per_b[b] = heavy
         vt = torch.as_tensor(np.ascontiguousarray(v, dtype=np.int64)).to(self.dev)
         stale = vt != (c - 1)
@@ -228,7 +237,18 @@ class FloorModel:
         p = pj // w.n_items
         sp = stale[p]
         items = int(torch.unique(vt[p[sp]] * w.n_items + (pj[sp] % w.n_items)).numel())
-        return 12 * n + 8 * w.K * w.n_users + 4 * w.K * (users + items), n
+        merged = w.n_users
+        words = 0
+        if self.skip:
+            assert c == self.last_c + 1, "the work-list floor needs every clock in order"
+            self.last_c = c
+            idle = torch.ones(w.n_users, dtype=torch.bool, device=self.dev)
+            idle[active] = False
+            skipped = int((idle & (c - self.chg >= w.s + 2)).sum())
+            merged = w.n_users - skipped
+            words = 4 * w.n_users
+            self.chg[active] = c
+        return 12 * n + 8 * w.K * merged + words + 4 * w.K * (users + items), n
 
 
 def _model_launches(w, c):
@@ -328,8 +348,8 @@ def measure(args, w, dev, world, rank, local):
     for c in range(1, W + K + 1):
         v, clk = t.read_schedule()
         assert clk == c
+        fb, n = model.bytes(c, v)  # every clock: the work-list floor follows the rows' history
         if c > W:
-            fb, n = model.bytes(c, v)
             floors.append(fb)
             counts.append(n)
             stale += np.bincount(c - 1 - v, minlength=w.s + 1)[: w.s + 1]

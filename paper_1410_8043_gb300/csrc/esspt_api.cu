@@ -42,6 +42,11 @@ struct esspt_ctx {
   // beside the work kernel (created on first use, on the context's device).
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // Work-list path: last clock that changed each user row, and the last clock
+  // at which every idle row is still copied forward (after an INC or a
+  // sequential clock, whose writes are not tracked per row).
+  int32_t* chg = nullptr;
+  int32_t copy_all_until = 0;
 };
 
 namespace {
@@ -193,7 +198,7 @@ bool is_host_ptr(const void* p) {
 
 struct MfCarve {
   size_t rec_u, rec_j, rec_D, rec_dst, uoff, mb_base, item_cnt, item_rep, dR, worker, chunk, chunk_base, heavy, heavy_base, dL,
-      user_slot, rec_row, total;
+      user_slot, rec_row, chg, total;
   int64_t max_chunks, max_heavy, dR_rows, dL_rows;
 };
 
@@ -232,6 +237,8 @@ MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int
   // holds at most n_obs entries).
   k.user_slot = row_mode ? take(sizeof(int32_t) * n_users) : o;
   k.rec_row = row_mode ? take(sizeof(int32_t) * (n_obs + 4)) : o;
+  // Work-list path: the clock that last changed each user row.
+  k.chg = uses_work16(K) ? take(sizeof(int32_t) * n_users) : o;
   k.total = o;
   return k;
 }
@@ -356,6 +363,10 @@ esspt_status esspt_table_init(esspt_ctx* c, const float* rows) {
   c->clock = 1;
   c->acc_ready = false;
   c->sched_set = false;
+  if (c->chg) {  // every row is version 0's: unchanged since clock 0
+    ESSPT_CUDA(c, cudaMemsetAsync(c->chg, 0, sizeof(int32_t) * (size_t)c->n_users, c->st));
+    c->copy_all_until = 0;
+  }
   if (c->cfg.model != ESSPT_EXTERNAL) return run_schedule(c);
   return ESSPT_OK;
 }
@@ -405,6 +416,9 @@ esspt_status esspt_inc(esspt_ctx* c, int32_t worker, const int32_t* d_row_ids, c
   if (n < 0 || (n > 0 && (!d_row_ids || !d_deltas))) return fail(c, ESSPT_EINVAL, "bad row list");
   if ((s = ensure_acc(c)) != ESSPT_OK) return s;
   ESSPT_CUDA(c, launch_inc(slot_ptr(c, c->clock), c->n_rows, c->K, d_row_ids, d_deltas, n, c->status, c->st));
+  // INC changes rows the work-list path does not track: copy every idle row
+  // until the changed version has gone round the ring.
+  c->copy_all_until = std::max(c->copy_all_until, c->clock + c->s + 1);
   return ESSPT_OK;
 }
 
@@ -555,6 +569,13 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   c->dL = dL;
   c->chunk = b.chunk;
   c->heavy = b.heavy;
+  c->chg = nullptr;
+  if (uses_work16(c->K)) {
+    c->chg = reinterpret_cast<int32_t*>(w + k.chg);
+    ESSPT_CUDA(c, cudaMemsetAsync(c->chg, 0, sizeof(int32_t) * (size_t)n_users, c->st));
+    // rows changed before this load are not tracked
+    c->copy_all_until = c->clock + c->s + 1;
+  }
   c->mb_base = mbb;
   c->chunk_base = chb;
   c->heavy_base = hvb;
@@ -595,6 +616,9 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   a.lambda = lambda;
   a.cap = cap;
   a.sq_loss = d_sq_loss;
+  a.chg = c->chg;
+  a.clock = c->clock;
+  a.copy_all_until = c->copy_all_until;
   if (c->rowver) {
     // Row-granular SSP: refresh the rows read this clock; the kernels then
     // take each user's slot and each entry's item ring row from the refresh.
@@ -663,6 +687,8 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
     h.dL = c->dL;
     h.eta = eta;
     h.cap = cap;
+    h.chg = c->chg;
+    h.clock = c->clock;
     ESSPT_CUDA(c, launch_heavy_merge(h, c->st));
   }
   if (c->ev_after) ESSPT_CUDA(c, cudaEventRecord(c->ev_after, c->st));
@@ -731,6 +757,8 @@ esspt_status esspt_mf_sgd_clock_sequential(esspt_ctx* c, float eta, float lambda
   if (c->ev_before) ESSPT_CUDA(c, cudaEventRecord(c->ev_before, c->st));
   ESSPT_CUDA(c, launch_seq_clock(a, c->st));
   if (c->ev_after) ESSPT_CUDA(c, cudaEventRecord(c->ev_after, c->st));
+  // the sequential kernels' row writes are not tracked per row
+  c->copy_all_until = std::max(c->copy_all_until, c->clock + c->s + 1);
   c->acc_ready = true;
   return advance(c);
 }

@@ -96,6 +96,12 @@ struct SgdArgs {
   double* sq_loss;          // optional
   int32_t row_mode;         // row-granular SSP: per-user slots and per-entry ring rows
   const int32_t* user_slot; // [n_users] row mode: ring slot of each user's cached row
+  // Work-list path: chg[u] = last clock that changed user row u (written with
+  // every user row that changes); an idle row whose slot already holds its
+  // current value is not copied forward: clock > copy_all_until and
+  // clock - chg[u] >= nslots (unchanged over the whole ring).
+  int32_t* chg;
+  int32_t clock, copy_all_until;
 };
 
 // Chunks of heavy users: x = user, y = begin, z = end (relative), w = replica row in dL.
@@ -118,6 +124,8 @@ struct HeavyMergeArgs {
   float* dL;
   float eta;
   int32_t cap;
+  int32_t* chg;             // work-list path: set chg[user] = clock (see SgdArgs)
+  int32_t clock;
 };
 
 // Clock() merge of the item rows: R^c_j = R^base_j + eta s_j sum of replicas.

@@ -740,6 +740,7 @@ __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(Chun
         float sc = a.eta;
         if (a.cap > 0 && n > a.cap) sc = a.eta * capped_scale(a.cap, n);
         st_stream_if(outq + (int64_t)u * K4 + r, f4_axpy(sc, g, lb), pol, on);
+        if (r == 0 && a.chg != nullptr) a.chg[u] = a.clock;
       }
     }
     m_it.x = __shfl_down_sync(0xffffffffu, m_it.x, kW16Unit);
@@ -757,7 +758,9 @@ __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(Chun
 // Forward copy of the users with no entry in minibatch b (version c-1 row to
 // version c), on the work-list path.  One warp per 32 consecutive users: their
 // entry counts come from two coalesced offset loads, and the warp copies the
-// rows of the idle ones, all loads of a unit in flight before the stores.
+// rows of the idle ones, all loads of a unit in flight before the stores.  A
+// row unchanged over the last s+2 clocks is skipped: the ring slot of version
+// c last held version c-(s+2), which is already its value.
 #ifndef ESSPT_COPY_BATCH
 #define ESSPT_COPY_BATCH 8
 #endif
@@ -773,10 +776,15 @@ __global__ void __launch_bounds__(256, 4) user_copy_kernel(SgdArgs a) {
   const uint64_t pol = policy_evict_first();
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const bool may_skip = a.chg != nullptr && a.clock > a.copy_all_until;
   for (int64_t u0 = warp * 32; u0 < a.n_users; u0 += nwarps * 32) {
     const int64_t u = u0 + lane;
     bool idle = false;
-    if (u < a.n_users) idle = __ldg(a.uoff + u + 1) == __ldg(a.uoff + u);
+    if (u < a.n_users) {
+      idle = __ldg(a.uoff + u + 1) == __ldg(a.uoff + u);
+      // unchanged over the whole ring: the slot of version c already holds it
+      if (idle && may_skip && a.clock - ld_stream_i32(a.chg + u, pol) >= a.nslots) idle = false;
+    }
     const unsigned mask = __ballot_sync(0xffffffffu, idle);
     if (mask == 0u) continue;
     // rows 2q + h of the unit, q = 0..15, in batches
@@ -899,6 +907,7 @@ __global__ void __launch_bounds__(256) heavy_merge_kernel(HeavyMergeArgs a) {
       const float4 b = ring4[(int64_t)a.slot_base * slot4 + (int64_t)hv.x * K4 + q];
       ring4[(int64_t)a.slot_out * slot4 + (int64_t)hv.x * K4 + q] = f4_axpy(sc, acc, b);
     }
+    if (lane == 0 && a.chg != nullptr) a.chg[hv.x] = a.clock;
   }
 }
 

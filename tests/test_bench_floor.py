@@ -39,6 +39,32 @@ def test_floor_model_matches_brute_force():
         assert m.bytes(c, v) == _brute_floor(w, d, wp, mb, c, v)
 
 
+def test_floor_model_work_list_skips_unchanged_idle_rows():
+    """On the work-list path (K 36..64) an idle user row unchanged over the last
+    s+2 clocks is not merged; every user has a 4-byte change-clock word."""
+    import bench
+    from gen.workloads import Workload
+
+    N, M, K, P, F, s = 150, 30, 40, 3, 4, 1
+    d = make_mf_data(n_users=N, n_items=M, n_obs=400, K=K, seed=8, truth_rank=2)
+    wp = shard_users(N, P, 9)
+    mb = minibatch_labels(400, F, 10)
+    w = Workload("t", N, M, 400, K=K, P=P, F=F, s=s, model="ssp", clocks=12, eta=0.01, lam=0.05, cap=0)
+    m = bench.FloorModel(w, d, wp, mb)
+    rng = np.random.default_rng(1)
+    chg = np.zeros(N, np.int64)
+    for c in range(1, 13):
+        v = rng.integers(max(0, c - 1 - s), c, size=P).astype(np.int32)
+        got = m.bytes(c, v)
+        base, n = _brute_floor(w, d, wp, mb, c, v)
+        active = np.zeros(N, bool)
+        active[d.i[mb == (c - 1) % F]] = True
+        skipped = int(np.sum(~active & (c - chg >= s + 2)))
+        assert skipped > 0 or c < s + 2
+        chg[active] = c
+        assert got == (base - 8 * K * skipped + 4 * N, n), c
+
+
 def test_model_launch_counts():
     import bench
     from gen import workload

@@ -361,3 +361,31 @@ def test_short_workspaces_are_refused():
     with pytest.raises(E.EssptError) as ei:
         t.mf_sgd_clock(0.01, 0.05)
     assert ei.value.status in (E.ESTATE,)
+
+
+@pytest.mark.parametrize("K", [40, 64])
+def test_idle_rows_skipped_across_the_ring(K):
+    """Work-list path, many clocks at s = 1 and 6 minibatches: most user rows
+    are idle for more than s+2 clocks in a row, so their forward copy is
+    skipped (the ring slot already holds them).  Every clock against the
+    oracle; then an INC on an idle row must survive the following clocks."""
+    E = _esspt()
+    N, M = 600, 80
+    d = make_mf_data(n_users=N, n_items=M, n_obs=3000, K=K, seed=K + 7, user_dist="zipf", user_a=1.2,
+                     truth_rank=3, truth_var=0.5, noise_var=0.1, init_var=0.05)
+    P, F, s = 4, 6, 1
+    wp, mb = shard_users(N, P, 3), minibatch_labels(3000, F, 4)
+    pair = Pair(d, wp, mb, P=P, s=s, F=F, model="ssp", eta=0.02, lam=0.05)
+    _run(pair, 14, obj_rtol=1e-5)
+    # an idle user in the coming clocks: INC its row at clock 15, which must
+    # stay in every later version (no skip may bring back an older copy)
+    coming = set(d.i[np.isin(mb, [(c - 1) % F for c in range(15, 21)])].tolist())
+    u = next(x for x in range(N) if x not in coming)
+    delta = np.full((1, K), 0.25, np.float32)
+    before = pair.t.read_table(14).cpu().numpy()[u].copy()
+    pair.t.inc(0, [u], delta)
+    for c in range(15, 21):
+        pair.t.mf_sgd_clock(pair.eta, pair.lam, 0)
+        got = pair.t.read_table(c).cpu().numpy()[u]
+        np.testing.assert_allclose(got, before + 0.25, rtol=0, atol=1e-6)
+    pair.t.poll()
