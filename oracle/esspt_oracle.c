@@ -8,8 +8,9 @@
  *     max(0, c-1-s) <= v_p(c) <= c-1, and s = 0 gives v = c-1: the BSP
  *     clock differential v - c = -1 of Fig. 1;
  *   - SSP lazy pull refreshes a worker's whole cached table only when it
- *     would otherwise break the bound ("waits until the last minute",
- *     Sec. 2.2), at a seeded per-worker phase phi_p in [0, s];
+ *     would otherwise break the bound (the SSP worker of Sec. 2.2 defers its
+ *     refresh as long as the bound allows), at a seeded per-worker phase phi_p
+ *     in [0, s];
  *   - ESSP eager push: the server's push of version c-1 reaches worker p
  *     after a delay of delta_{p,c} ~ Geometric(p) clocks clamped to
  *     [0, min(max_delay, s)]; the read version never goes backwards;

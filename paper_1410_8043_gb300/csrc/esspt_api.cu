@@ -47,6 +47,7 @@ struct esspt_ctx {
   // sequential clock, whose writes are not tracked per row).
   int32_t* chg = nullptr;
   int32_t copy_all_until = 0;
+  int32_t* hot_item = nullptr;   // work-list path: [F][kHot] hot items of each minibatch
 };
 
 namespace {
@@ -198,7 +199,7 @@ bool is_host_ptr(const void* p) {
 
 struct MfCarve {
   size_t rec_u, rec_j, rec_D, rec_dst, uoff, mb_base, item_cnt, item_rep, dR, worker, chunk, chunk_base, heavy, heavy_base, dL,
-      user_slot, rec_row, chg, total;
+      user_slot, rec_row, chg, hot_item, total;
   int64_t max_chunks, max_heavy, dR_rows, dL_rows;
 };
 
@@ -239,6 +240,7 @@ MfCarve mf_carve(int64_t n_obs, int64_t n_users, int64_t n_items, int32_t F, int
   k.rec_row = row_mode ? take(sizeof(int32_t) * (n_obs + 4)) : o;
   // Work-list path: the clock that last changed each user row.
   k.chg = uses_work16(K) ? take(sizeof(int32_t) * n_users) : o;
+  k.hot_item = uses_hot(K) ? take(sizeof(int32_t) * (size_t)F * kHot) : o;
   k.total = o;
   return k;
 }
@@ -515,6 +517,7 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   b.heavy_base = reinterpret_cast<int64_t*>(w + k.heavy_base);
   b.max_chunks = k.max_chunks;
   b.light_items = uses_work16(c->K);
+  b.hot_item = uses_hot(c->K) ? reinterpret_cast<int32_t*>(w + k.hot_item) : nullptr;
   b.max_heavy = k.max_heavy;
   b.scratch = d_scratch;
   b.scratch_bytes = scratch_bytes;
@@ -570,6 +573,7 @@ esspt_status esspt_mf_load(esspt_ctx* c, const int32_t* d_i, const int32_t* d_j,
   c->chunk = b.chunk;
   c->heavy = b.heavy;
   c->chg = nullptr;
+  c->hot_item = b.hot_item;
   if (uses_work16(c->K)) {
     c->chg = reinterpret_cast<int32_t*>(w + k.chg);
     ESSPT_CUDA(c, cudaMemsetAsync(c->chg, 0, sizeof(int32_t) * (size_t)n_users, c->st));
@@ -618,6 +622,7 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   a.sq_loss = d_sq_loss;
   a.chg = c->chg;
   a.clock = c->clock;
+  a.hot_item = c->hot_item ? c->hot_item + (int64_t)b * kHot : nullptr;
   a.copy_all_until = c->copy_all_until;
   if (c->rowver) {
     // Row-granular SSP: refresh the rows read this clock; the kernels then

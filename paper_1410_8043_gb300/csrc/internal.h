@@ -53,6 +53,15 @@ inline bool uses_work16(int32_t K) { return K > 32 && K <= 64; }
 #define ESSPT_FORK_COPY 0
 #endif
 constexpr bool kForkCopy = ESSPT_FORK_COPY != 0;
+// Work-list path: the kHot items with the most entries of each minibatch have
+// their updates summed per warp in shared memory and added to the replica
+// rows once per warp instead of once per entry (0 = off).  An entry of hot
+// slot h carries rec_dst = -1 - h.
+#ifndef ESSPT_W16_HOT
+#define ESSPT_W16_HOT 2
+#endif
+constexpr int kHot = ESSPT_W16_HOT;
+inline bool uses_hot(int32_t K) { return kHot > 0 && uses_work16(K); }
 constexpr int kCopyBlocksPerSm = kForkCopy ? 1 : 8;
 constexpr int kWorkBlocksPerSm = kForkCopy ? 2 : 8;
 
@@ -102,6 +111,7 @@ struct SgdArgs {
   // clock - chg[u] >= nslots (unchanged over the whole ring).
   int32_t* chg;
   int32_t clock, copy_all_until;
+  const int32_t* hot_item;  // [kHot] work-list path: item of each hot slot of minibatch b, -1 if unused
 };
 
 // Chunks of heavy users: x = user, y = begin, z = end (relative), w = replica row in dL.
@@ -229,6 +239,7 @@ struct LayoutBuild {
   int64_t* heavy_base;  // [F+1]
   int64_t max_chunks, max_heavy;
   bool light_items;     // also list every user with 1..kHeavy entries (work-list path)
+  int32_t* hot_item;    // [F][kHot] work-list path with kHot > 0: the hot items of each minibatch
   // scratch
   void* scratch;
   size_t scratch_bytes;

@@ -6,6 +6,7 @@
 // the chunk and heavy-user lists and the replica rows of popular items and
 // heavy users.
 #include <algorithm>
+#include <vector>
 
 #include <cub/device/device_radix_sort.cuh>
 #include <cub/device/device_scan.cuh>
@@ -163,9 +164,12 @@ __global__ void item_reps_kernel(const int32_t* __restrict__ item_cnt, int64_t n
 // Replica row of every entry's item update: entry t (position within its
 // minibatch) of item j adds into replica (t mod replicas of j): replica 0 is
 // row j, replica r > 0 row n_items + item_rep[j] + r - 1.
+// With hot_item (work-list path, kHot > 0) an entry of hot slot h of its
+// minibatch gets -1 - h instead.
 __global__ void dst_kernel(const uint32_t* __restrict__ key, const int64_t* __restrict__ mb_base,
                            const int32_t* __restrict__ rec_j, const int32_t* __restrict__ item_rep, int64_t n_obs,
-                           int64_t n_users, int64_t n_items, int32_t* __restrict__ rec_dst) {
+                           int64_t n_users, int64_t n_items, const int32_t* __restrict__ hot_item,
+                           int32_t* __restrict__ rec_dst) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < n_obs; k += stride) {
     const int64_t b = (int64_t)key[k] / n_users;
@@ -173,8 +177,34 @@ __global__ void dst_kernel(const uint32_t* __restrict__ key, const int64_t* __re
     const int32_t j = rec_j[k];
     const int32_t e0 = item_rep[j], e1 = item_rep[j + 1];  // extra replicas of j: e1 - e0 (reps - 1)
     const int32_t r = (int32_t)(t & (int64_t)(e1 - e0));    // reps is a power of two
-    rec_dst[k] = r == 0 ? j : (int32_t)(n_items + e0 + r - 1);
+    int32_t d = r == 0 ? j : (int32_t)(n_items + e0 + r - 1);
+    if (hot_item != nullptr)
+      for (int h = 0; h < kHot; ++h)
+        if (hot_item[b * kHot + h] == j) d = -1 - h;
+    rec_dst[k] = d;
   }
+}
+
+// The kHot items with the most entries of each minibatch (at least 2), most
+// popular first, ties by id; -1 for unused slots.  Host side, at setup.
+cudaError_t build_hot(const LayoutBuild& b, cudaStream_t st) {
+  if (kHot <= 0 || b.hot_item == nullptr) return cudaSuccess;
+  const size_t FM = (size_t)b.F * (size_t)b.n_items;
+  std::vector<int32_t> cnt(FM), hot((size_t)b.F * kHot, -1), idx((size_t)b.n_items);
+  cudaError_t e = cudaMemcpyAsync(cnt.data(), b.item_cnt, sizeof(int32_t) * FM, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return e;
+  for (int32_t mb = 0; mb < b.F; ++mb) {
+    const int32_t* c = cnt.data() + (size_t)mb * b.n_items;
+    for (int64_t j = 0; j < b.n_items; ++j) idx[j] = (int32_t)j;
+    const int64_t h = std::min<int64_t>(kHot, b.n_items);
+    std::partial_sort(idx.begin(), idx.begin() + h, idx.end(),
+                      [c](int32_t x, int32_t y) { return c[x] != c[y] ? c[x] > c[y] : x < y; });
+    for (int64_t r = 0; r < h && c[idx[r]] >= 2; ++r) hot[(size_t)mb * kHot + r] = idx[r];
+  }
+  e = cudaMemcpyAsync(b.hot_item, hot.data(), sizeof(int32_t) * hot.size(), cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  return e;
 }
 
 // A staged minibatch against the loaded one: every user id, item id and
@@ -322,8 +352,9 @@ cudaError_t build_layout(const LayoutBuild& b, cudaStream_t st) {
   if ((e = cub::DeviceScan::ExclusiveSum(cub_tmp, tb, ireps, b.item_rep, (int)(b.n_items + 1), st)) != cudaSuccess)
     return e;
   if (b.n_obs == 0) return cudaSuccess;
+  if ((e = build_hot(b, st)) != cudaSuccess) return e;
   dst_kernel<<<blocks_for(b.n_obs), 256, 0, st>>>(key_out, b.mb_base, b.rec_j, b.item_rep, b.n_obs, b.n_users,
-                                                  b.n_items, b.rec_dst);
+                                                  b.n_items, kHot > 0 ? b.hot_item : nullptr, b.rec_dst);
   return cudaGetLastError();
 }
 

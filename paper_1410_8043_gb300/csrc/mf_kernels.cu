@@ -541,7 +541,7 @@ __global__ void __launch_bounds__(256, ESSPT_USERS32_MINB) sgd_users32_kernel(Sg
 // memory one pair ahead by cp.async, and each warp walks one contiguous range
 // of items, balanced by entries plus kItemCost per item.
 #ifndef ESSPT_WORK16_MINB
-#define ESSPT_WORK16_MINB 3
+#define ESSPT_WORK16_MINB 4
 #endif
 #ifndef ESSPT_W16_ITEMCOST
 #define ESSPT_W16_ITEMCOST 6
@@ -553,6 +553,10 @@ constexpr int32_t kNoItem = -2;   // metadata of a slot past the warp's range
 __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(ChunkArgs c) {
   const SgdArgs& a = c.a;
   __shared__ __align__(16) float4 stage[8][2][2][32];  // [warp][buffer][read row, base row][half * 16 + slice]
+#if ESSPT_W16_HOT > 0
+  // per warp and lane: the summed updates of the minibatch's hot items
+  __shared__ __align__(16) float4 hacc[8][kHot][32];
+#endif
   const int lane = threadIdx.x & 31;
   const int wib = threadIdx.x >> 5;
   const int h = lane >> 4;      // half: its own item
@@ -608,6 +612,9 @@ __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(Chun
     flush_loss(a.sq_loss, 0.f, lane);
     return;
   }
+#if ESSPT_W16_HOT > 0
+  for (int hs = 0; hs < kHot; ++hs) hacc[wib][hs][lane] = f4_zero();
+#endif
 
   // Item metadata: the current unit in lanes [0, 16), the next in [16, 32).
   int4 m_it = make_int4(0, 0, 0, kNoItem);
@@ -711,10 +718,16 @@ __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(Chun
           gL.y += ev * rr.y;
           gL.z += ev * rr.z;
           gL.w += ev * rr.w;
-          red_add_v4_if(dRq + dsts[e] * a.dR_ld,
-                        make_float4(ev * Lv.x - a.lambda * rr.x, ev * Lv.y - a.lambda * rr.y,
-                                    ev * Lv.z - a.lambda * rr.z, ev * Lv.w - a.lambda * rr.w),
-                        on && (kFull || e < cnt));
+          const float4 dv = make_float4(ev * Lv.x - a.lambda * rr.x, ev * Lv.y - a.lambda * rr.y,
+                                        ev * Lv.z - a.lambda * rr.z, ev * Lv.w - a.lambda * rr.w);
+          const bool val = on && (kFull || e < cnt);
+#if ESSPT_W16_HOT > 0
+          const int32_t dd = dsts[e];
+          red_add_v4_if(dRq + dd * a.dR_ld, dv, val && dd >= 0);
+          if (val && dd < 0) hacc[wib][-1 - dd][lane] = f4_add(hacc[wib][-1 - dd][lane], dv);
+#else
+          red_add_v4_if(dRq + dsts[e] * a.dR_ld, dv, val);
+#endif
         }
       };
       for (int32_t sidx = 0; sidx < steps; ++sidx) {
@@ -752,6 +765,26 @@ __global__ void __launch_bounds__(256, ESSPT_WORK16_MINB) sgd_work16_kernel(Chun
     __syncwarp();
   }
   cp_async_wait_all();
+#if ESSPT_W16_HOT > 0
+  // Hot items: both halves' sums, added once into a replica row of the item
+  // (the warp index picks among its replicas).
+  __syncwarp();
+  {
+    const int64_t wg = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t n_items_all = a.n_rows - a.n_users;
+    float4* dR4 = reinterpret_cast<float4*>(a.dR);
+    for (int hs = 0; hs < kHot; ++hs) {
+      const int32_t j = __ldg(a.hot_item + hs);
+      const float4 v = f4_add(hacc[wib][hs][lane], hacc[wib][hs][lane ^ 16]);
+      if (j >= 0 && h == 0 && on) {
+        const int32_t e0 = __ldg(a.item_rep + j), e1 = __ldg(a.item_rep + j + 1);
+        const int32_t rr = (int32_t)(wg & (int64_t)(e1 - e0));  // replicas are a power of two
+        const int64_t row = rr == 0 ? (int64_t)j : n_items_all + e0 + rr - 1;
+        red_add_v4(dR4 + row * a.dR_ld + r, v);
+      }
+    }
+  }
+#endif
   flush_loss(a.sq_loss, loss, lane);
 }
 
@@ -913,11 +946,12 @@ __global__ void __launch_bounds__(256) heavy_merge_kernel(HeavyMergeArgs a) {
 
 // Clock() merge of the item rows (Sec. 2.1 additive updates, Sec. 4 server
 // clock): R^c_j = R^base_j + eta s_j sum of j's replica rows; replicas
-// cleared.  One thread per (item, float4 slice).  Replica 0 of item j is row
-// j of dR, so the common single-replica item needs no index load before its
-// data loads: every load of a thread is issued at once.  With do_schedule the
+// cleared.  Each thread merges U (item, float4 slice) pairs.  Replica 0 of
+// item j is row j of dR, so the common single-replica item needs no index
+// load before its data loads: every load of a thread is issued at once.  With do_schedule the
 // first P threads also compute the next clock's read versions (the SGD
 // kernels of this clock, the only readers of v, have finished).
+template <int U>  // (item, slice) pairs per thread per round, the loads of all in flight
 __global__ void __launch_bounds__(256) item_merge_kernel(ItemMergeArgs a) {
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t nth = (int64_t)gridDim.x * blockDim.x;
@@ -930,10 +964,6 @@ __global__ void __launch_bounds__(256) item_merge_kernel(ItemMergeArgs a) {
   // n_items * K/4 < 2^31 (checked at load), so the (item, slice) split is a
   // 32-bit division
   const int64_t total = (int64_t)a.n_items * K4;
-#ifndef ESSPT_MERGE_U
-#define ESSPT_MERGE_U 8
-#endif
-  constexpr int U = ESSPT_MERGE_U;  // (item, slice) pairs per thread per round, loads of all in flight
   for (int64_t x0 = tid; x0 < total; x0 += U * nth) {
     float4 first[U], base[U];
     int32_t e0[U], e1[U], cnt[U];
@@ -945,14 +975,8 @@ __global__ void __launch_bounds__(256) item_merge_kernel(ItemMergeArgs a) {
       const int32_t q = (int32_t)((uint32_t)x - j * (uint32_t)K4);
       row[k] = ((int64_t)a.n_users + j) * K4 + q;
       dofs[k] = (int64_t)j * a.dR_ld + q;
-#ifdef ESSPT_MERGE_STREAM
-      const uint64_t pol = policy_evict_first();
-      first[k] = ld_stream(dR4 + dofs[k], pol);
-      base[k] = ld_stream(ring4 + (int64_t)a.slot_base * slot4 + row[k], pol);
-#else
       first[k] = dR4[dofs[k]];
       base[k] = ring4[(int64_t)a.slot_base * slot4 + row[k]];
-#endif
       e0[k] = __ldg(a.item_rep + j);
       e1[k] = __ldg(a.item_rep + j + 1);
       cnt[k] = __ldg(a.item_cnt + j);
@@ -1055,7 +1079,7 @@ cudaError_t launch_sgd_chunks(const ChunkArgs& c, cudaStream_t st) { return disp
 // One resident wave of sgd_work16_kernel; its warps balance the items among
 // themselves.
 #ifndef ESSPT_W16_CARVEOUT
-#define ESSPT_W16_CARVEOUT 25
+#define ESSPT_W16_CARVEOUT 50
 #endif
 cudaError_t launch_sgd_work16(const ChunkArgs& c, cudaStream_t st) {
   if (c.n_chunks <= 0) return cudaSuccess;
@@ -1097,11 +1121,14 @@ cudaError_t launch_heavy_merge(const HeavyMergeArgs& a, cudaStream_t st) {
 cudaError_t launch_item_merge(const ItemMergeArgs& a, cudaStream_t st) {
   const int64_t work = std::max<int64_t>((int64_t)a.n_items * (a.K >> 2), a.do_schedule ? a.sched.P : 0);
   if (work <= 0) return cudaSuccess;
-  // One thread per (item, slice): every thread's loads are independent, so
-  // the whole merge is one set of in-flight requests rather than a
-  // grid-stride chain of dependent ones.
-  const int64_t blocks = std::min<int64_t>((work + 255 * ESSPT_MERGE_U) / (256 * ESSPT_MERGE_U), (int64_t)1 << 30);
-  item_merge_kernel<<<(unsigned)blocks, 256, 0, st>>>(a);
+  // Every thread's loads are independent, so the whole merge is one set of
+  // in-flight requests.  Large tables take 8 (item, slice) pairs per thread;
+  // small ones one, which keeps enough threads to fill the GPU.
+  if (work >= ((int64_t)1 << 23)) {
+    item_merge_kernel<8><<<(unsigned)std::min<int64_t>((work + 2047) / 2048, (int64_t)1 << 30), 256, 0, st>>>(a);
+  } else {
+    item_merge_kernel<1><<<(unsigned)((work + 255) / 256), 256, 0, st>>>(a);
+  }
   return cudaGetLastError();
 }
 
