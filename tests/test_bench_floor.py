@@ -76,3 +76,61 @@ def test_model_launch_counts():
     w = workload("mid_vap")
     assert bench._model_launches(w, 1) == 2 and bench._model_launches(w, 10) == 2
     assert bench._model_launches(w.with_(s=9), 10) == 3
+
+
+def test_host_minibatches_are_disjoint_views_of_one_buffer(monkeypatch):
+    """bench.py's end-to-end leg exports every minibatch into views of one host
+    buffer: each view has the size and dtype the export call checks, and no
+    two views overlap."""
+    import torch
+
+    import bench
+    from gen.workloads import Workload
+
+    class CpuBuffer:
+        kind = "test"
+
+        def __init__(self, n_int32):
+            self.tensor = torch.zeros(n_int32, dtype=torch.int32)
+            self.closed = False
+
+        def close(self):
+            self.closed = True
+
+    sizes = {0: 7, 2: 0, 3: 13}
+    w = Workload("t", 5, 4, 20, K=8, P=2, F=4, s=1, model="ssp", clocks=3, eta=0.01, lam=0.05, cap=0)
+
+    class FakeTable:
+        n_users = w.n_users
+
+        def mf_minibatch_size(self, b):
+            return sizes[b]
+
+        def mf_export_minibatch(self, b, out):
+            u, j, D, uoff = out
+            n = sizes[b]
+            assert u.numel() == j.numel() == D.numel() == n and uoff.numel() == w.n_users + 1
+            assert u.dtype == j.dtype == uoff.dtype == torch.int32 and D.dtype == torch.float32
+            assert all(x.is_contiguous() for x in out)
+            u.fill_(100 + b)
+            j.fill_(200 + b)
+            D.fill_(0.5 + b)
+            uoff.copy_(torch.arange(w.n_users + 1, dtype=torch.int32) + b)
+            return out
+
+    monkeypatch.setattr(bench, "HostBuffer", CpuBuffer)
+    out, buf = bench._export_host_minibatches(FakeTable(), w, sorted(sizes))
+    assert buf.tensor.numel() == sum(3 * n + w.n_users + 1 for n in sizes.values())
+    spans = []
+    base = buf.tensor.data_ptr()
+    for b, (u, j, D, uoff) in out.items():
+        assert bool((u == 100 + b).all()) and bool((j == 200 + b).all()) and bool((D == 0.5 + b).all())
+        assert uoff.tolist() == [x + b for x in range(w.n_users + 1)]
+        for x in (u, j, D, uoff):
+            if x.numel() == 0:  # an empty view has no address to check
+                continue
+            lo = x.data_ptr() - base
+            spans.append((lo, lo + 4 * x.numel()))
+            assert 0 <= lo and lo + 4 * x.numel() <= 4 * buf.tensor.numel()
+    spans.sort()
+    assert all(a[1] <= b[0] for a, b in zip(spans, spans[1:]))
