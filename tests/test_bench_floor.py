@@ -134,3 +134,14 @@ def test_host_minibatches_are_disjoint_views_of_one_buffer(monkeypatch):
             assert 0 <= lo and lo + 4 * x.numel() <= 4 * buf.tensor.numel()
     spans.sort()
     assert all(a[1] <= b[0] for a, b in zip(spans, spans[1:]))
+
+
+def test_committed_profiles_match_the_kernel_source():
+    """The bench line's roofline.traffic comes from the committed ncu summary
+    of each headline kernel, and only while the summary's source hash equals
+    the kernels' current source: both summaries must be current."""
+    import bench
+
+    assert bench._profiled_traffic("sgd_work16_kernel", "large") == 7995646720.0
+    assert bench._profiled_traffic("sgd_users32_kernel", "mid") == 692899584.0
+    assert bench._profiled_traffic("sgd_users32_kernel", "large") is None
