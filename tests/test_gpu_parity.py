@@ -141,6 +141,66 @@ def test_heavy_users_chunk_path(K):
     _run(pair, 4, obj_rtol=1e-5)
 
 
+@pytest.mark.parametrize("K", [16, 48, 64, 100, 132])
+def test_popular_items_with_extra_replicas(K):
+    """Items popular enough for extra replica rows (one per 2048 entries of
+    their largest minibatch, a power of two, at most 64), here 1 to 64 of
+    them, beside heavy users, idle users and (for K = 48, 64) the two hot
+    items that the work-list kernel sums per warp.  The item merge must add
+    every replica and clear it for the next clock."""
+    n = 400_000
+    d = make_mf_data(n_users=3000, n_items=40, n_obs=n, K=K, seed=11, user_dist="zipf", user_a=1.2,
+                     item_dist="zipf", item_a=1.5, truth_rank=4, truth_var=0.5, noise_var=0.1, init_var=0.05)
+    F = 2
+    mb = minibatch_labels(n, F, 12)
+    mx = np.max([np.bincount(d.j[mb == b], minlength=40) for b in range(F)], axis=0)
+    want = -(-mx // 2048)
+    assert want.max() > 32 and ((want > 1) & (want <= 8)).sum() >= 3  # the cap of 64 and small counts
+    users = np.bincount(d.i[mb == 0], minlength=3000)
+    assert (users > 96).sum() >= 10 and (users == 0).sum() >= 1
+    pair = Pair(d, shard_users(3000, 6, 13), mb, P=6, s=2, F=F, model="essp", eta=0.005, lam=0.05, cap=20)
+    _run(pair, 5, obj_rtol=1e-5)
+    assert min(pair.moved) > 10 * TOL
+
+
+@pytest.mark.parametrize("K", [16, 64, 100])
+def test_rows_that_no_entry_names(K):
+    """Users and items that no entry names keep their initial rows, bit for bit,
+    in every version, through more clocks than the ring has slots (so the
+    work-list path also skips their forward copies)."""
+    d = make_mf_data(n_users=400, n_items=90, n_obs=12000, K=K, seed=21, item_dist="zipf", item_a=1.0,
+                     truth_rank=4, truth_var=0.5, noise_var=0.1, init_var=0.05)
+    d.i = (d.i % 390).astype(np.int32)  # users 390..399 and items 80..89 have no entries
+    d.j = (d.j % 80).astype(np.int32)
+    P, F, s = 4, 3, 1
+    pair = Pair(d, shard_users(400, P, 22), minibatch_labels(12000, F, 23), P=P, s=s, F=F, model="ssp",
+                eta=0.01, lam=0.05, cap=10)
+    x0 = np.concatenate([d.L0, d.R0])
+    quiet = np.r_[390:400, 400 + 80:400 + 90]
+    for c in range(1, 9):
+        pair.step(obj_rtol=1e-5)
+        np.testing.assert_array_equal(pair.t.read_table(c).cpu().numpy()[quiet], x0[quiet])
+    assert min(pair.moved) > 10 * TOL
+
+
+@pytest.mark.parametrize("K", [16, 64, 100])
+@pytest.mark.parametrize("shape", ["one_item", "one_user"])
+def test_single_item_or_single_user(shape, K):
+    """Every entry on one item (a hot item with the most replicas) or on one
+    user (one heavy user split into many chunks)."""
+    if shape == "one_item":
+        N, M, n = 600, 1, 150_000
+    else:
+        N, M, n = 1, 300, 20_000
+    d = make_mf_data(n_users=N, n_items=M, n_obs=n, K=K, seed=31, truth_rank=4, truth_var=0.5, noise_var=0.1,
+                     init_var=0.05)
+    P, F = 3, 2
+    pair = Pair(d, shard_users(N, P, 32), minibatch_labels(n, F, 33), P=P, s=1, F=F, model="essp", eta=0.005,
+                lam=0.05, cap=20)
+    _run(pair, 5, obj_rtol=1e-5)
+    assert min(pair.moved) > 10 * TOL
+
+
 def test_empty_and_degenerate():
     """No entries at all; P larger than the number of users; one worker."""
     E = _esspt()
