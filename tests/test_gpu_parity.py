@@ -104,6 +104,31 @@ def test_tiny_workload_every_clock(model):
     assert min(pair.moved) > 10 * TOL
 
 
+@pytest.mark.parametrize("p,max_delay,s", [(0.3, 6, 8), (0.9, 1, 4), (1.0, 3, 3), (0.05, 8, 8), (0.5, 5, 2)])
+def test_essp_delay_law_parameters(p, max_delay, s):
+    """ESSP with other push probabilities and delay clamps than the workloads'
+    (Geometric(0.7), clamp 3): the read versions of 64 workers over 40 clocks
+    equal the oracle's rule bit for bit, within the clamp min(max_delay, s)
+    and spread over several staleness values."""
+    E = _esspt()
+    P, seed = 64, 77
+    t = E.Table(8, 4, P, s, model="essp", essp_p=p, essp_max_delay=max_delay, seed=seed)
+    t.table_init(np.zeros((8, 4), np.float32))
+    want = _oracle_schedules(dict(n_users=1, n_items=1, K=1, P=P, s=s, F=1, model="essp", seed=seed, essp_p=p,
+                                  essp_max_delay=max_delay), 40)
+    stale = set()
+    for c in range(1, 41):
+        v, clk = t.read_schedule()
+        assert clk == c
+        np.testing.assert_array_equal(v, want[c - 1], err_msg=f"clock {c}")
+        stale.update((c - 1 - v).tolist())
+        t.clock()
+    t.poll()
+    bound = 0 if p == 1.0 else min(max_delay, s)
+    assert max(stale) <= bound and len(stale) >= min(bound + 1, 5)
+    t.close()
+
+
 @pytest.mark.parametrize("K", [4, 8, 12, 16, 36, 52, 64, 100, 128, 132, 260])
 def test_row_widths_and_ragged_tail(K):
     """Every row-group shape (lanes per row, float4 per lane) and ragged K."""
@@ -240,11 +265,13 @@ def test_inc_then_sgd_in_one_clock():
     np.testing.assert_allclose(g, pair.o.table() + extra, rtol=0, atol=TOL * 4)
 
 
-def test_get_inc_clock_semantics():
+@pytest.mark.parametrize("n_rows,K,n_ids", [(37, 8, 9), (37, 100, 9), (5003, 64, 2000), (301, 512, 150)])
+def test_get_inc_clock_semantics(n_rows, K, n_ids):
     """GET returns the worker's read version; INC + CLOCK add into the next
-    version; versions outside the window are refused."""
+    version; versions outside the window are refused.  Row widths from 8 to
+    the largest (512), and id lists that span many blocks."""
     E = _esspt()
-    n_rows, K, P, s = 37, 8, 3, 2
+    P, s = 3, 2
     t = E.Table(n_rows, K, P, s, model="ssp", phased=True, seed=11)
     x = np.random.default_rng(1).normal(size=(n_rows, K)).astype(np.float32)
     t.table_init(x)
@@ -254,14 +281,14 @@ def test_get_inc_clock_semantics():
         v, clk = t.read_schedule()
         assert clk == c
         for p in range(P):
-            ids = rng.integers(0, n_rows, size=9).astype(np.int32)
+            ids = rng.integers(0, n_rows, size=n_ids).astype(np.int32)
             rows, ver = t.get(p, ids, want_version=True)
             assert ver == v[p]
             np.testing.assert_array_equal(rows.cpu().numpy(), hist[ver][ids].astype(np.float32))
         acc = hist[-1].copy()
         for p in range(P):
-            ids = rng.integers(0, n_rows, size=6).astype(np.int32)
-            dl = rng.normal(size=(6, K)).astype(np.float32)
+            ids = rng.integers(0, n_rows, size=2 * n_ids // 3).astype(np.int32)
+            dl = rng.normal(size=(ids.size, K)).astype(np.float32)
             t.inc(p, ids, dl)
             np.add.at(acc, ids, dl.astype(np.float64))
         t.clock()

@@ -63,6 +63,44 @@ def test_vap_tiny_every_clock(v0):
     t.close()
 
 
+@pytest.mark.parametrize("K,v0", [(48, 0.6), (64, 0.6), (100, 0.8)])
+def test_vap_wide_rows_every_clock(K, v0):
+    """VAP on the work-list path (K = 48, 64) and on the one-slice-per-lane
+    kernel (K = 100), Zipf items, a hot-row cap: schedule bit-exact and every
+    parameter within tolerance for 12 clocks, reads of every staleness 0..3."""
+    from gen import make_mf_data, minibatch_labels, shard_users
+
+    E = _esspt()
+    N, M, n, P, F, s = 500, 60, 20000, 7, 4, 3
+    d = make_mf_data(n_users=N, n_items=M, n_obs=n, K=K, seed=3, item_dist="zipf", item_a=1.0, truth_rank=4,
+                     truth_var=0.5, noise_var=0.1, init_var=0.05)
+    wp, mb = shard_users(N, P, 5), minibatch_labels(n, F, 6)
+    eta, lam, cap = 0.01, 0.05, 12
+    t = E.Table(N + M, K, P, s, model="vap", vap_v0=v0)
+    t.mf_load(d.i, d.j, d.D, mb, wp, N, F)
+    t.table_init(np.concatenate([d.L0, d.R0]))
+    cfg = OracleConfig(n_users=N, n_items=M, K=K, P=P, s=s, F=F, model="vap", phased=True, seed=8043, eta=eta,
+                       lam=lam, cap=cap, vap_v0=v0)
+    o = Oracle(cfg, d.i, d.j, d.D, mb, wp, d.L0, d.R0)
+    seen = set()
+    for c in range(1, 13):
+        v_gpu, clk = t.read_schedule()
+        assert clk == c
+        o.clock()
+        v_or = o.schedule()
+        norms, bound = o.vap_norms()
+        for k in range(1, min(s, c - 1) + 1):
+            if 0.0 < bound < 1e20:
+                assert abs(norms[k] - bound) > MARGIN * bound, (c, k, norms[k], bound)
+        np.testing.assert_array_equal(v_gpu, v_or, err_msg=f"clock {c}")
+        seen.add(int(c - 1 - v_or[0]))
+        t.mf_sgd_clock(eta, lam, cap)
+        g = t.read_table(c).cpu().numpy().astype(np.float64)
+        assert _viol(g, o.table()) <= 0.0, f"clock {c}: max |err| {np.abs(g - o.table()).max():.3e}"
+    assert seen == {0, 1, 2, 3}
+    t.close()
+
+
 def test_vap_get_inc_clock_by_hand():
     """VAP on the generic GET/INC/CLOCK path with hand-set deltas (s = 2, v0 = 1):
     clock 1 adds 1/2 to row 0, clock 2 adds 1/4 to row 1, clock 3 adds 1/8 to
