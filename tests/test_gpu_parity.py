@@ -338,6 +338,41 @@ def test_external_schedule_and_errors():
     assert ei.value.status == E.ESTATE
 
 
+@pytest.mark.parametrize("K", [16, 64, 100])
+def test_external_schedule_random_versions(K):
+    """The MF clock under caller-chosen read versions: every worker draws its
+    own version anywhere in [max(0, c-1-s), c-1] each clock (not monotone, not
+    shared), with heavy users and popular items, so one clock gathers from
+    up to s+1 versions at once."""
+    E = _esspt()
+    N, M, n, P, F, s = 2000, 50, 120_000, 9, 3, 4
+    d = make_mf_data(n_users=N, n_items=M, n_obs=n, K=K, seed=41, user_dist="zipf", user_a=1.2,
+                     item_dist="zipf", item_a=1.5, truth_rank=4, truth_var=0.5, noise_var=0.1, init_var=0.05)
+    wp, mb = shard_users(N, P, 42), minibatch_labels(n, F, 43)
+    eta, lam, cap = 0.005, 0.05, 20
+    t = E.Table(N + M, K, P, s, model="external")
+    t.mf_load(d.i, d.j, d.D, mb, wp, N, F)
+    t.table_init(np.concatenate([d.L0, d.R0]))
+    o = Oracle(OracleConfig(n_users=N, n_items=M, K=K, P=P, s=s, F=F, model="external", eta=eta, lam=lam, cap=cap),
+               d.i, d.j, d.D, mb, wp, d.L0, d.R0)
+    rng = np.random.default_rng(44)
+    spread = []
+    for c in range(1, 11):
+        v = rng.integers(max(0, c - 1 - s), c, size=P).astype(np.int32)
+        spread.append(len(set(v.tolist())))
+        t.set_schedule(v)
+        t.mf_sgd_clock(eta, lam, cap)
+        o.clock(v_ext=v)
+        g = t.read_table(c).cpu().numpy().astype(np.float64)
+        assert _max_violation(g, o.table()) <= 0.0, f"clock {c}: max |err| {np.abs(g - o.table()).max():.3e}"
+    t.poll()
+    assert max(spread) == s + 1
+    gs, gp = t.mf_objective(10, lam)
+    os_, op = o.objective()
+    assert abs(gs - os_) <= 1e-5 * abs(os_) and abs(gp - op) <= 1e-5 * abs(op)
+    t.close()
+
+
 def test_mf_load_rejects_bad_indices():
     E = _esspt()
     t = E.Table(30, 4, 2, 1)

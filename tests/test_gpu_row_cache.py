@@ -69,6 +69,20 @@ def test_row_cache_heavy_users(K):
               cap=50, clocks=4)
 
 
+@pytest.mark.parametrize("K", [64, 100])
+def test_row_cache_popular_items(K):
+    """Popular items with many replica rows (and, at K = 64, the hot items that
+    the work-list kernel sums per warp) while each worker reads its own cached
+    version of every row; 6 clocks, sparse minibatches so rows age."""
+    n = 200_000
+    d = make_mf_data(n_users=2000, n_items=40, n_obs=n, K=K, seed=51, user_dist="zipf", user_a=1.2,
+                     item_dist="zipf", item_a=1.5, truth_rank=4, truth_var=0.5, noise_var=0.1, init_var=0.05)
+    mb = minibatch_labels(n, 3, 52)
+    mx = np.max([np.bincount(d.j[mb == b], minlength=40) for b in range(3)], axis=0)
+    assert (-(-mx // 2048)).max() > 8  # at least one item with 16 replica rows
+    _run_pair(d, shard_users(2000, 5, 53), mb, P=5, s=2, F=3, eta=0.005, lam=0.05, cap=20, clocks=6)
+
+
 def test_row_cache_get_by_hand():
     """GET under the row-granular cache, s = 1, rows of 4 values, X0 = 0:
       clock 1: worker 0 reads row 0 (not cached: version 0) and adds 1 to it;
