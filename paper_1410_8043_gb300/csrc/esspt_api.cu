@@ -38,10 +38,6 @@ struct esspt_ctx {
   int4 *chunk = nullptr, *heavy = nullptr;
   std::vector<int64_t> mb_base, chunk_base, heavy_base;
   cudaEvent_t ev_before = nullptr, ev_after = nullptr;
-  // Work-list path: the forward copy of idle users runs on a second stream
-  // beside the work kernel (created on first use, on the context's device).
-  cudaStream_t side = nullptr;
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   // Work-list path: last clock that changed each user row, and the last clock
   // at which every idle row is still copied forward (after an INC or a
   // sequential clock, whose writes are not tracked per row).
@@ -343,12 +339,6 @@ esspt_status esspt_create(const esspt_config* cfg, void* d_workspace, size_t byt
 esspt_status esspt_destroy(esspt_ctx* c) {
   if (!c) return ESSPT_OK;
   cudaError_t e = cudaStreamSynchronize(c->st);
-  if (c->side) {
-    cudaStreamSynchronize(c->side);
-    cudaStreamDestroy(c->side);
-  }
-  if (c->ev_fork) cudaEventDestroy(c->ev_fork);
-  if (c->ev_join) cudaEventDestroy(c->ev_join);
   delete c;
   return e == cudaSuccess ? ESSPT_OK : ESSPT_ECUDA;
 }
@@ -657,24 +647,8 @@ esspt_status esspt_mf_sgd_clock(esspt_ctx* c, float eta, float lambda, int32_t c
   if (uses_work16(c->K)) {
     // Work-list path: users without entries are copied forward; every other
     // user (and every chunk of a heavy user) is one item of the work kernel.
-    // The copy is HBM streaming and the work kernel mostly L2 traffic, so the
-    // copy runs on a second stream beside it.
-    if (kForkCopy) {
-      if (!c->side) {
-        ESSPT_CUDA(c, cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking));
-        ESSPT_CUDA(c, cudaEventCreateWithFlags(&c->ev_fork, cudaEventDisableTiming));
-        ESSPT_CUDA(c, cudaEventCreateWithFlags(&c->ev_join, cudaEventDisableTiming));
-      }
-      ESSPT_CUDA(c, cudaEventRecord(c->ev_fork, c->st));
-      ESSPT_CUDA(c, cudaStreamWaitEvent(c->side, c->ev_fork, 0));
-      ESSPT_CUDA(c, launch_user_copy(a, c->side));
-      ESSPT_CUDA(c, cudaEventRecord(c->ev_join, c->side));
-      ESSPT_CUDA(c, launch_sgd_work16(ch, c->st));
-      ESSPT_CUDA(c, cudaStreamWaitEvent(c->st, c->ev_join, 0));
-    } else {
-      ESSPT_CUDA(c, launch_user_copy(a, c->st));
-      ESSPT_CUDA(c, launch_sgd_work16(ch, c->st));
-    }
+    ESSPT_CUDA(c, launch_user_copy(a, c->st));
+    ESSPT_CUDA(c, launch_sgd_work16(ch, c->st));
   } else {
     if (nch > 0) ESSPT_CUDA(c, launch_sgd_chunks(ch, c->st));
     ESSPT_CUDA(c, launch_sgd_users(a, c->st));

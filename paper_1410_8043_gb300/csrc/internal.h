@@ -46,13 +46,6 @@ constexpr int32_t kMaxRep = ESSPT_MAX_REP;
 // chunks of the heavy users, processed by one kernel, and the users without
 // entries are copied forward by a streaming kernel.
 inline bool uses_work16(int32_t K) { return K > 32 && K <= 64; }
-// Run the forward copy of idle users on a second stream beside the work
-// kernel (each then takes part of every SM: kernels sized by kCopyBlocksPerSm
-// and kWorkBlocksPerSm).
-#ifndef ESSPT_FORK_COPY
-#define ESSPT_FORK_COPY 0
-#endif
-constexpr bool kForkCopy = ESSPT_FORK_COPY != 0;
 // Work-list path: the kHot items with the most entries of each minibatch have
 // their updates summed per warp in shared memory and added to the replica
 // rows once per warp instead of once per entry (0 = off).  An entry of hot
@@ -62,8 +55,10 @@ constexpr bool kForkCopy = ESSPT_FORK_COPY != 0;
 #endif
 constexpr int kHot = ESSPT_W16_HOT;
 inline bool uses_hot(int32_t K) { return kHot > 0 && uses_work16(K); }
-constexpr int kCopyBlocksPerSm = kForkCopy ? 1 : 8;
-constexpr int kWorkBlocksPerSm = kForkCopy ? 2 : 8;
+// Resident blocks per SM that the launches of the forward copy and of the
+// work kernel ask for (the occupancy limit caps the second).
+constexpr int kCopyBlocksPerSm = 8;
+constexpr int kWorkBlocksPerSm = 8;
 
 // Row stride (in float4) of the item delta replicas: K rounded up to a whole
 // number of 32-byte sectors, so that a row's reductions touch the fewest sectors.
