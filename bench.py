@@ -266,7 +266,7 @@ def _stage_overlapped(t, w, host_mb, W, K, stream, copy_stream, loss_d, loss_h):
     """K clocks through the public API with host inputs: minibatch of clock
     c+1 is copied from pinned host memory on `copy_stream` while clock c runs
     on `stream`; each clock's squared loss is copied back to pinned host
-    memory.  Returns (h2d bytes, d2h bytes)."""
+    memory.  Returns (start event on `stream`, h2d bytes, d2h bytes)."""
     import torch
 
     F = w.F
