@@ -205,6 +205,25 @@ def test_essp_stationary_staleness_closed_form():
     assert abs(st.mean() - 0.327729) < 5 * st.std() / np.sqrt(n) * 3
 
 
+@pytest.mark.parametrize("p", [0.5, 0.3])
+def test_essp_stationary_staleness_other_laws(p):
+    """The same closed form for other push probabilities, with the clamp at 8
+    out of the way: P(st >= k) = (1-p)^(k(k+1)/2), since st_c >= k needs
+    d_c >= k and st_{c-1} >= k-1."""
+    P, C, q = 1024, 1200, 1.0 - p
+    cfg = OracleConfig(n_users=1, n_items=1, K=1, P=P, s=8, F=1, model="essp", seed=8043, essp_p=p,
+                       essp_max_delay=8)
+    sched = _run_schedule(cfg, C)
+    c = np.arange(1, C + 1)[:, None]
+    st = (c - 1 - sched)[30:].ravel()
+    n = st.size
+    ge = np.array([q ** (k * (k + 1) / 2) for k in range(7)])
+    want = ge[:6] - ge[1:7]  # P(st = k), k = 0..5
+    got = np.bincount(st, minlength=9)[:6]
+    sigma = np.sqrt(n * want * (1 - want))
+    assert (np.abs(got - n * want) < 5 * sigma).all(), (got / n, want)
+
+
 def test_essp_delay_thresholds_exact():
     """The ESSP delay rule's 32-bit thresholds are floor(0.3^k 2^32) for the
     Geometric(0.7) delay (failures before the first success), computed here
@@ -215,6 +234,23 @@ def test_essp_delay_thresholds_exact():
     want = [int(Fraction(3, 10) ** k * 2 ** 32) for k in (1, 2, 3)]
     assert want == [1288490188, 386547056, 115964116]
     assert essp_thresholds(cfg) == want
+
+
+@pytest.mark.parametrize("p", ["0.5", "0.3", "0.05", "0.9", "1"])
+def test_essp_delay_thresholds_other_laws(p):
+    """The same thresholds for other push probabilities and a clamp of 8:
+    floor((1-p)^k 2^32) from the decimal p in exact rational arithmetic
+    (p = 1 gives no delay: every threshold 0; p = 0.5 gives 2^(32-k))."""
+    from oracle import essp_thresholds
+
+    cfg = OracleConfig(n_users=1, n_items=1, K=1, P=1, s=8, F=1, model="essp", essp_p=float(p), essp_max_delay=8)
+    q = 1 - Fraction(p)
+    want = [int(q ** k * 2 ** 32) for k in range(1, 9)]
+    assert essp_thresholds(cfg) == want
+    if p == "0.5":
+        assert want == [2 ** (32 - k) for k in range(1, 9)]
+    if p == "1":
+        assert want == [0] * 8
 
 
 def test_essp_clamped_by_s():
