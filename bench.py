@@ -34,15 +34,26 @@ METRIC = "SGD ratings/sec per clock on 1 GB300; achieved HBM GB/s vs peak"
 UNIT = "ratings/s"
 
 
+def kernel_code_digest(text: str) -> str:
+    """First 16 hex digits of the SHA-256 of a CUDA source's code: comments
+    removed and every run of whitespace made one space, so that editing a
+    comment keeps the digest and any change to the code changes it."""
+    import hashlib
+    import re
+
+    code = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    code = re.sub(r"//[^\n]*", " ", code)
+    code = " ".join(code.split())
+    return hashlib.sha256(code.encode()).hexdigest()[:16]
+
+
 def _profiled_traffic(kernel: str, workload: str):
     """DRAM bytes per launch of `kernel` on `workload` from its committed ncu
     summary profiles/<kernel>_<workload>.md, or None when there is none or the
-    kernel source changed since the capture."""
-    import hashlib
-
+    kernels' code changed since the capture."""
     src = os.path.join(ROOT, "paper_1410_8043_gb300", "csrc", "mf_kernels.cu")
     try:
-        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        digest = kernel_code_digest(open(src).read())
     except OSError:
         return None
     for path in [os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")]:
@@ -53,7 +64,7 @@ def _profiled_traffic(kernel: str, workload: str):
             if ":" in line and not line.startswith(("|", "#", " ", "`")):
                 k, _, v = line.partition(":")
                 fields[k.strip()] = v.strip()
-        if fields.get("kernel_source_sha256_16") == digest and "traffic_bytes_per_launch" in fields:
+        if fields.get("kernel_code_sha256_16") == digest and "traffic_bytes_per_launch" in fields:
             return float(fields["traffic_bytes_per_launch"])
     return None
 

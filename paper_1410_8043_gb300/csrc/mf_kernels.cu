@@ -1,8 +1,15 @@
 // Matrix-factorisation SGD on the version ring (Sec. 3.1 updates under the
-// SSP / ESSP read schedule).  One clock is:
+// SSP / ESSP read schedule).  One clock is, for rows of 36..64 values (the
+// work-list path):
+//   user_copy_kernel    users without entries: row of version c-1 carried to
+//                       version c, unless unchanged over the whole ring;
+//   sgd_work16_kernel   every user with entries (its row of version c,
+//                       written once) and every chunk of a very active one;
+// and for other row widths:
 //   sgd_chunks_kernel   entries of very active users, in chunks (if any);
 //   sgd_users_kernel    every other user: its row of version c, written once
 //                       (sgd_users32_kernel for rows of 68..128 values);
+// then, for both:
 //   heavy_merge_kernel  rows of the very active users (if any);
 //   item_merge_kernel   the Clock() merge of the item rows.
 // Item-row (and heavy-user) deltas are summed, unscaled, into zero-initialised

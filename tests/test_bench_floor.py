@@ -138,10 +138,21 @@ def test_host_minibatches_are_disjoint_views_of_one_buffer(monkeypatch):
 
 def test_committed_profiles_match_the_kernel_source():
     """The bench line's roofline.traffic comes from the committed ncu summary
-    of each headline kernel, and only while the summary's source hash equals
-    the kernels' current source: both summaries must be current."""
+    of each headline kernel, and only while the summary's code digest equals
+    that of the kernels' current source: both summaries must be current."""
     import bench
 
     assert bench._profiled_traffic("sgd_work16_kernel", "large") == 7995646720.0
     assert bench._profiled_traffic("sgd_users32_kernel", "mid") == 692899584.0
     assert bench._profiled_traffic("sgd_users32_kernel", "large") is None
+
+
+def test_kernel_code_digest_ignores_comments_only():
+    """The digest that ties a profile to the kernels' code ignores comments and
+    layout, and changes with any token of code."""
+    import bench
+
+    base = "int f(int x) {\n  return x + 1;  // one more\n}\n"
+    assert bench.kernel_code_digest(base) == bench.kernel_code_digest(
+        "/* header */\nint f(int x) {\n    return x + 1;\n}\n")
+    assert bench.kernel_code_digest(base) != bench.kernel_code_digest(base.replace("x + 1", "x + 2"))
